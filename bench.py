@@ -1,0 +1,355 @@
+"""Benchmark: translated tokens/s at batch 1, GS-Jacobi (b=5) vs greedy AR, on the Marian-sized
+bf16 model (6+6 layers, d=512, 8 heads, FFN 2048 SiLU, V=58101) over 256 synthetic source
+sentences of 8..64 ids with max_len = 2 * src_len, plus the decode kernel's HBM roofline.
+
+One step = encode + decode of all 256 sentences, one after the other (batch 1).
+  value : tokens/s with source ids resident in device memory, timed with CUDA events on the
+          library stream (pd_encode_device / pd_decode_device), L2 flushed between steps.
+  e2e   : the same through the host API (pd_encode / pd_decode: ids copied in, tokens copied
+          out, every call synchronous), wall clock.
+Multi-GPU: replicas (every rank decodes the full sentence set; weak scaling).
+``--impl reference`` times the CPU oracle (numpy float64) on a bounded sample instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+WORKLOAD = synth.MARIAN_GS
+METRIC = "translated tokens/s at batch 1, GS-Jacobi vs greedy AR; HBM GB/s % of peak"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def pass_bytes(spec: synth.ModelSpec, L_keys: int, n_src: int, rows: int) -> int:
+    """Algorithmic HBM bytes of one decoder pass: every decoder-layer and LM-head parameter
+    once, the self-attention keys/values of positions 0..L_keys-1 and the cross keys/values
+    of the n_src source positions once, and the K/V written for the pass's rows."""
+    d, f, V, Ld = spec.d_model, spec.d_ff, spec.vocab, spec.n_dec_layers
+    es = 2 if spec.dtype == synth.DTYPE_BF16 else 4
+    layer = 3 * d * d + 3 * d + d * d + d + d * d + d + d * d + d + 2 * d * f + f + d + 6 * d
+    weights = Ld * layer + V * d
+    kv = Ld * 2 * d * (L_keys + n_src) + Ld * 2 * d * rows
+    return es * (weights + kv)
+
+
+def decode_bytes(spec, n_src, trace):
+    """Sum of pass_bytes over the passes of one decode (from its trace)."""
+    tot = 0
+    for row in trace:
+        i, blk = row["block_start"], row["block_len"]
+        tot += pass_bytes(spec, i - 1 + blk, n_src, blk)
+    return tot
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index),
+                                          f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and --impl reference)
+# ---------------------------------------------------------------------------------------------
+
+def oracle_tokens_per_s(weights, sentences, budget_s):
+    from oracle import decode as od
+    from oracle import model as om
+    model = om.Model(WORKLOAD.spec, weights.tensors)
+    tokens, t0, used = 0, time.perf_counter(), []
+    for k, src in enumerate(sentences):
+        step = od.model_step(model, src)
+        r = od.gs_jacobi(step, WORKLOAD.max_len(len(src)), WORKLOAD.b)
+        tokens += len(r.tokens)
+        used.append(k)
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return tokens / dt, tokens, dt, used
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    weights = synth.make_weights(WORKLOAD.spec, seed=WORKLOAD.weight_seed)
+    sents = WORKLOAD.sentences()
+    # each step: GS-Jacobi (b=5) of the next sentence of the workload by the float64 oracle
+    order = sorted(range(len(sents)), key=lambda k: len(sents[k]))[:args.warmup + args.steps]
+    for k in order[:args.warmup]:
+        oracle_tokens_per_s(weights, [sents[k]], 0)
+    tok, dt = 0, 0.0
+    for k in order[args.warmup:]:
+        _, t, d, _ = oracle_tokens_per_s(weights, [sents[k]], 0)
+        tok += t
+        dt += d
+    v = tok / dt
+    cores = os.cpu_count()
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD.name, "sample": "one sentence per step, the "
+                       "shortest sentences of the 256 (CPU oracle is slow)"},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{args.steps} sentences, GS-Jacobi b=5, numpy float64, "
+                                       f"BLAS threads = all {cores} cores"},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------------------------
+
+def run_gpu(args):
+    import torch
+    import paper_2305_10427_gb300 as pkg
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+
+    if not os.path.exists(pkg.LIB_PATH):
+        from paper_2305_10427_gb300 import build
+        build.build(force=False)
+
+    spec = WORKLOAD.spec
+    weights = synth.make_weights(spec, seed=WORKLOAD.weight_seed)
+    sents = WORKLOAD.sentences()
+    n_s = len(sents)
+    max_src = max(len(s) for s in sents)
+    max_tgt = max(WORKLOAD.max_len(len(s)) for s in sents)
+    stream = torch.cuda.Stream()
+    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt), weights.blob,
+                      stream=stream.cuda_stream)
+
+    offs = np.cumsum([0] + [len(s) for s in sents])
+    d_src = torch.tensor(np.concatenate(sents), dtype=torch.int32, device="cuda")
+    d_y = torch.zeros((n_s, max_tgt), dtype=torch.int32, device="cuda")
+    d_info = torch.zeros((n_s, 4), dtype=torch.int32, device="cuda")
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
+    params = {m: [pkg.Decoder.params(m, WORKLOAD.max_len(len(s)), b=WORKLOAD.b)
+                  for s in sents] for m in ("gs_jacobi", "greedy")}
+
+    def device_step(method, ev=None):
+        for k in range(n_s):
+            if ev is not None:
+                ev[k][0].record(stream)
+            dec.encode_device(d_src.data_ptr() + 4 * int(offs[k]), len(sents[k]))
+            if ev is not None:
+                ev[k][1].record(stream)
+            dec.decode_device(params[method][k], d_y[k].data_ptr(), d_info[k].data_ptr())
+            if ev is not None:
+                ev[k][2].record(stream)
+
+    def timed(method, steps, warmup):
+        for _ in range(warmup):
+            device_step(method)
+        torch.cuda.synchronize()
+        total_ms, dec_ms, launches0 = 0.0, 0.0, dec.launch_count
+        tokens = 0
+        for _ in range(steps):
+            flush.fill_(1)                     # evict L2 (256 MB > 129 MB) between steps
+            ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n_s)]
+            torch.cuda.synchronize()
+            if dist is not None:
+                dist.barrier()
+            with torch.cuda.stream(stream):
+                device_step(method, ev)
+            torch.cuda.synchronize()
+            total_ms += ev[0][0].elapsed_time(ev[-1][2])
+            dec_ms += sum(e[1].elapsed_time(e[2]) for e in ev)
+            info = d_info.cpu().numpy()
+            assert (info[:, 2] == 0).all(), "decode reported a failure"
+            tokens += int(info[:, 0].sum())
+        return tokens, total_ms, dec_ms, dec.launch_count - launches0, d_info.cpu().numpy()
+
+    def max_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t)
+        return float(t.item())
+
+    # greedy AR reference point (same kernels, one position per pass)
+    g_tok, g_ms, g_dec_ms, _, g_info = timed("greedy", args.steps, args.warmup)
+    g_ms = max_over_ranks(g_ms)
+    greedy_tps = sum_over_ranks(g_tok) / (g_ms / 1e3)
+
+    with Clocks(local) as clk:
+        tok, ms, dec_ms, launches, info = timed("gs_jacobi", args.steps, args.warmup)
+    ms_max = max_over_ranks(ms)
+    tps = sum_over_ranks(tok) / (ms_max / 1e3)
+
+    # roofline of the decode kernel: algorithmic bytes from the traces of one step
+    total_bytes, passes = 0, 0
+    toks = []
+    for k, s in enumerate(sents):
+        dec.encode(s)
+        r = dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b, trace=True)
+        assert r.n_iters == int(info[k, 1])
+        total_bytes += decode_bytes(spec, len(s), r.trace)
+        passes += r.n_iters
+        toks.append(len(r.tokens))
+    dec_s_per_step = dec_ms / args.steps / 1e3
+    achieved = total_bytes / dec_s_per_step / 1e9
+    peak, peak_kind = peaks()
+
+    # end to end through the host API
+    e2e_tok, h2d, d2h = 0, 0, 0
+    for _ in range(args.warmup):
+        for k, s in enumerate(sents[:8]):
+            dec.encode(s)
+            dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        for k, s in enumerate(sents):
+            dec.encode(s)
+            r = dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b)
+            e2e_tok += len(r.tokens)
+            h2d += 4 * len(s)
+            d2h += 4 + 16 + 4 * len(r.tokens)      # encode status, decode info, tokens
+    torch.cuda.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0)
+    e2e_tps = sum_over_ranks(e2e_tok) / e2e_s
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        v, t, d, used = oracle_tokens_per_s(weights, [sents[k] for k in
+                                                      sorted(range(n_s), key=lambda k:
+                                                             len(sents[k]))], args.cpu_budget)
+        cpu = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"{len(used)} shortest sentences of the 256 ({t} tokens, {d:.1f} s), "
+                         f"GS-Jacobi b=5, numpy float64, BLAS threads = all cores"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": tps, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded N(0,0.02) weights, uniform random source ids",
+            "config": {"workload": WORKLOAD.name, "sentences_per_step": n_s,
+                       "timing": "CUDA events on the library stream; L2 flushed (256 MB write) "
+                                 "between steps; replicas across GPUs"},
+            "greedy": {"value": greedy_tps, "unit": "tokens/s",
+                       "gs_jacobi_speedup": tps / greedy_tps},
+            "passes_per_token": passes / max(1, sum(toks)),
+            "us_per_pass": 1e6 * dec_s_per_step / max(1, passes),
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "kernel": "decode_kernel<bf16>", "peak_kind": peak_kind},
+            "e2e": {"value": e2e_tps, "unit": "tokens/s", "h2d_bytes_per_step": h2d // args.steps,
+                    "d2h_bytes_per_step": d2h // args.steps},
+            "gpu_launches": launches,
+            "clocks": clk.summary(),
+        }
+        if cpu is not None:
+            line["cpu_baseline"] = cpu
+        print(json.dumps(line), flush=True)
+    dec.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,162 @@
+/*
+ * pd.h — C ABI of a single-GPU (GB300, sm_103a) parallel decoder for encoder-decoder
+ * translation transformers, after "Accelerating Transformer Inference for Translation via
+ * Parallel Decoding" (Santilli et al., arXiv 2305.10427).
+ *
+ * The paper states the problem as: given a source sentence x = (x_1..x_n), return
+ * y = (y_1..y_m) with y_i = argmax p_theta(y_i | y_1..y_{i-1}, x) (Section 3.1, Eq. 1-2),
+ * and solves that triangular system (Eq. 3-4) with Jacobi (Algorithm 1), GS-Jacobi
+ * (Algorithm 2) or Hybrid GS-Jacobi (Algorithm 3) fixed-point iterations, drafts initialised
+ * to PAD (Section 3.3, InitT) and stopped when a block no longer changes (Eq. 5, StopC).
+ *
+ * Conventions for every entry point:
+ *  - Host pointers are plain CPU memory owned by the caller; "d_" pointers are device memory
+ *    of the context's GPU owned by the caller.  The library never keeps a caller pointer.
+ *  - The library allocates all of its device memory in pd_create, sized for the capacities in
+ *    pd_config; pd_encode / pd_decode allocate nothing (pd_debug_logits is the one exception,
+ *    a test-only call).
+ *  - Arguments are checked before anything is launched; a bad argument returns PD_EINVAL and
+ *    leaves the context unchanged.  A CUDA failure returns PD_ECUDA.  pd_last_error() gives a
+ *    one-line reason for the last failure on that context.  No C++ exception crosses the ABI.
+ *  - A context is used by one host thread at a time.  All work is issued on the context's
+ *    stream (the one passed to pd_create, or a stream the library creates).
+ */
+#ifndef PD_H
+#define PD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  PD_OK = 0,
+  PD_EINVAL = -1,    /* bad argument or unsupported configuration */
+  PD_ENOMEM = -2,    /* device allocation failed in pd_create */
+  PD_ECUDA = -3,     /* a CUDA runtime call or kernel failed */
+  PD_ENOTCONV = -4,  /* the pass budget (pd_decode_params.max_passes) ran out first */
+  PD_ENAN = -5,      /* a NaN appeared in the logits */
+  PD_ESTATE = -6,    /* pd_decode before any successful pd_encode */
+  PD_ETIMEOUT = -7   /* a device-side wait gave up (the kernel returned instead of hanging) */
+} pd_status;
+
+typedef enum {
+  PD_GREEDY = 0,            /* Eq. 2: one position per decoder pass */
+  PD_JACOBI = 1,            /* Algorithm 1: the whole sentence is one block */
+  PD_GS_JACOBI = 2,         /* Algorithm 2: blocks of b positions, solved in order */
+  PD_HYBRID_GS_JACOBI = 3   /* Algorithm 3: GS-Jacobi up to h, EOS exit, greedy tail */
+} pd_method;
+
+typedef enum { PD_ACT_RELU = 0, PD_ACT_SILU = 1, PD_ACT_GELU = 2 } pd_activation;
+typedef enum { PD_DTYPE_F32 = 0, PD_DTYPE_BF16 = 1 } pd_dtype;
+
+/* Model structure and capacities.  The paper runs a base (d=512, 6+6 layers) and a big
+ * (d=1024, 12+12 layers) transformer (Section 4.1, "Model Configuration"); everything it
+ * leaves to the model library is fixed here: token embedding scaled by sqrt(d_model) and
+ * tied with the output projection (no logits bias), sinusoidal ([sin | cos], frequency
+ * 10000^(-2k/d), from position 0) or learned positions, post-LN (x = LN(x + f(x))) or pre-LN
+ * (x = x + f(LN(x)) with embedding and final LayerNorms), attention scale 1/sqrt(d_head).
+ * Supported: d_model and d_ff multiples of 256, d_model / n_heads in {32, 64, 128},
+ * n_enc_layers and n_dec_layers in [1, 16]. */
+typedef struct {
+  int d_model, n_heads, d_ff, n_enc_layers, n_dec_layers, vocab;
+  int activation;    /* pd_activation */
+  int pre_ln;        /* 0: post-LN, 1: pre-LN */
+  int learned_pos;   /* 0: sinusoidal, 1: learned table of max_pos rows */
+  int max_pos;       /* rows of the learned position table */
+  int dtype;         /* pd_dtype: storage of every parameter; activations are fp32 */
+  int pad_id, eos_id, bos_id;
+  float ln_eps;
+  int max_src_len;   /* capacity: longest source sentence pd_encode accepts */
+  int max_tgt_len;   /* capacity: largest max_len pd_decode accepts */
+} pd_config;
+
+typedef struct pd_ctx pd_ctx;
+
+/* Size in bytes of the weight blob for cfg: every parameter in the documented order (token
+ * embedding [V,d]; learned positions [max_pos,d] if any; pre-LN only: encoder and decoder
+ * embedding-LN and final-LN gain/bias; then per encoder layer wqkv [3d,d], bqkv, wo [d,d],
+ * bo, ln1 g/b, w1 [f,d], b1, w2 [d,f], b2, ln2 g/b; then per decoder layer wqkv, bqkv, wo, bo,
+ * ln1 g/b, wq_c [d,d], bq_c, wkv_c [2d,d], bkv_c, wo_c [d,d], bo_c, ln2 g/b, w1, b1, w2, b2,
+ * ln3 g/b), row-major, linear maps stored [out, in], elements float32 or bfloat16 bits.
+ * Returns 0 for an invalid cfg. */
+size_t pd_weights_nbytes(const pd_config* cfg);
+
+/* Create a context on the current CUDA device: validate cfg, allocate every device buffer for
+ * the capacities in cfg, and upload the weight blob (host memory, nbytes =
+ * pd_weights_nbytes(cfg)).  stream is a cudaStream_t (NULL: the library creates its own).
+ * On success *out owns all device memory until pd_destroy. */
+pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, void* stream,
+                    pd_ctx** out);
+
+/* Copy the device weights back in blob order (dst host memory of nbytes). */
+pd_status pd_export_weights(pd_ctx* ctx, void* dst, size_t nbytes);
+
+/* Run the encoder once for a source sentence x_1..x_n (host int32 ids, 1 <= n_src <=
+ * max_src_len, each in [0, vocab)) and cache the cross-attention keys and values of every
+ * decoder layer; only the decoder runs per iteration (Fig. 1; Section 4.1 caches keys and
+ * values).  Synchronous. */
+pd_status pd_encode(pd_ctx* ctx, const int32_t* src, int n_src);
+
+/* As pd_encode, with the ids already in device memory (d_src); asynchronous on the context
+ * stream (ids are not range-checked; out-of-range ids are clamped on the device). */
+pd_status pd_encode_device(pd_ctx* ctx, const int32_t* d_src, int n_src);
+
+typedef struct {
+  int method;       /* pd_method */
+  int b;            /* block size for GS-Jacobi / hybrid (>= 1); ignored by greedy, jacobi */
+  int max_len;      /* 1 <= max_len <= max_tgt_len; for jacobi / gs_jacobi it is the known
+                       target length m of Section 4.1 */
+  int h;            /* hybrid: parallel part up to position h (0 = max_len) */
+  int stop_at_eos;  /* greedy / jacobi / gs_jacobi: end the returned y at the first EOS */
+  int max_passes;   /* 0 = no limit; else stop with PD_ENOTCONV after this many passes */
+} pd_decode_params;
+
+/* One decoder pass of the trace (DDGviz-style, Section 3.5): pass number (1-based), block
+ * start position i (1-based), block length, number of leading block positions whose new
+ * token equals the previous draft, StopC (Eq. 5) flag, index of the first EOS in the new
+ * block tokens (-1 if none). */
+typedef struct {
+  int32_t step, block_start, block_len, n_converged, stop, eos_idx;
+} pd_trace_step;
+
+/* Decode the sentence last given to pd_encode.  Outputs (host): y[0..*n_y) = y_1..y_m
+ * (capacity max_len), *n_iters = decoder passes (encoder excluded).  Optional trace (NULL to
+ * skip): trace[trace_cap], trace_tokens[trace_cap][max_len] (row t holds the pass's
+ * block_len new tokens), trace_probs same shape (softmax probability of each argmax token);
+ * *n_trace = rows written (min(passes, trace_cap)).  Synchronous.  Returns PD_ESTATE without
+ * a prior pd_encode. */
+pd_status pd_decode(pd_ctx* ctx, const pd_decode_params* p, int32_t* y, int* n_y, int* n_iters,
+                    pd_trace_step* trace, int32_t* trace_tokens, float* trace_probs,
+                    int trace_cap, int* n_trace);
+
+/* As pd_decode, asynchronous on the context stream, outputs in device memory: d_y[max_len]
+ * and d_info[4] = {n_y, n_iters, status, n_trace}.  Parameters are checked on the host. */
+pd_status pd_decode_device(pd_ctx* ctx, const pd_decode_params* p, int32_t* d_y,
+                           int32_t* d_info);
+
+/* Test-only: teacher-forced logits of one decoder pass over the input tokens y_in[0..len)
+ * at positions 0..len-1 (row t scores position t+1, Eq. 1) for the sentence last encoded.
+ * logits: host float32 [len][vocab].  Allocates a temporary device buffer; overwrites the
+ * decoder's key/value cache. */
+pd_status pd_debug_logits(pd_ctx* ctx, const int32_t* y_in, int len, float* logits);
+
+/* The context's cudaStream_t. */
+void* pd_stream(pd_ctx* ctx);
+
+/* Number of the library's kernel launches issued on this context so far. */
+int64_t pd_launch_count(const pd_ctx* ctx);
+
+/* One-line reason for the last failure on ctx ("" if none); valid until the next call. */
+const char* pd_last_error(const pd_ctx* ctx);
+
+/* Free every device buffer and the context (NULL is a no-op). */
+void pd_destroy(pd_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PD_H */

@@ -1,0 +1,863 @@
+// pd.cu — kernels and C ABI of the GB300 parallel decoder (see include/pd.h).
+//
+// Execution model.  One persistent, cooperatively launched kernel per pd_encode and per
+// pd_decode call: one 512-thread CTA per SM.  pd_decode's kernel runs the whole decoding
+// loop on the device — every decoder pass (embedding, Ld x {QKV, self-attention, O-proj,
+// cross-Q, cross-attention, cross-O, FFN1, FFN2}, LM head with fused argmax) and the
+// fixed-point commit that advances the block — with grid barriers between phases and no
+// host round trip per pass.  The pass loop is bounded by Proposition 1 (at most m passes)
+// and by the optional pass budget; every device wait is bounded in time.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "pd.h"
+#include "pd_device.cuh"
+
+namespace pd {
+
+template <typename W>
+struct KParams {
+  Dims D;
+  const ModelW<W>* mw;      // device copy of the weight-pointer table
+  Bufs<W> B;
+  int n_src;                // encoder length (cross-attention keys)
+  const int* enc_tok;       // encoder input ids (device)
+  int debug_len;            // > 0: one teacher-forced pass over dbg_tok, logits out
+  float* logits;            // [debug_len][V]
+  DecState init;            // method, b, max_len, h, stop_at_eos, max_passes
+  int32_t* out_y;           // [max_len]
+  int32_t* out_info;        // {n_y, n_iters, status, n_trace}
+};
+
+struct SmemLayout {
+  size_t xs, part, scratch, commit, total;
+};
+
+__host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
+  SmemLayout L;
+  const int kmax = D.d > D.f ? D.d : D.f;
+  L.xs = 0;
+  L.part = L.xs + ((size_t)kMTile * kmax * wsize + 15) / 16 * 16;
+  L.scratch = L.part + (size_t)kWarps * kMTile * sizeof(Partial);
+  L.commit = L.scratch + (size_t)kWarps * (128 + D.rows + 4) * sizeof(float);
+  L.total = L.commit + (size_t)(D.max_tgt + 1) * 2 * sizeof(int) + 64;
+  return L;
+}
+
+// ------------------------------------------------------------------------------------------
+// one decoder pass over M rows (input tokens tok[0..M) at positions pos0..pos0+M-1)
+// ------------------------------------------------------------------------------------------
+
+template <typename W>
+__device__ bool decoder_pass(const KParams<W>& P, int M, int pos0, const int* tok,
+                             unsigned& tgt, unsigned char* smem) {
+  const Dims& D = P.D;
+  const Bufs<W>& B = P.B;
+  const ModelW<W>& mw = *P.mw;
+  int* status = &B.st->status;
+  const SmemLayout SL = smem_layout(D, sizeof(W));
+  float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
+
+  embed_phase<W>(D, mw.embed, mw.pos, D.pre_ln ? mw.dec_lne_g : nullptr,
+                 D.pre_ln ? mw.dec_lne_b : nullptr, tok, pos0, M, B.ra);
+  if (!grid_barrier(B.bar, tgt, status)) return false;
+
+  for (int l = 0; l < D.Ld; ++l) {
+    const DecLayerW<W>& L = mw.dec[l];
+    W* kc = B.kself + (size_t)l * D.max_tgt * D.d;
+    W* vc = B.vself + (size_t)l * D.max_tgt * D.d;
+    W* kx = B.kcross + (size_t)l * D.max_src * D.d;
+    W* vx = B.vcross + (size_t)l * D.max_src * D.d;
+    // sublayer inputs: pre-LN normalises with the sublayer's own LN and keeps the raw
+    // residual; post-LN normalises with the previous sublayer's LN and that normalised row
+    // is the residual (the first sublayer takes the embedding as is).
+    const W *g1, *b1;
+    float *st1;
+    const float* res1;
+    if (D.pre_ln) { g1 = L.ln1g; b1 = L.ln1b; st1 = nullptr; res1 = B.ra; }
+    else if (l == 0) { g1 = nullptr; b1 = nullptr; st1 = nullptr; res1 = B.ra; }
+    else { g1 = mw.dec[l - 1].ln3g; b1 = mw.dec[l - 1].ln3b; st1 = B.xa; res1 = B.xa; }
+
+    GemmArgs<W> g{};
+    g.M = M; g.N = 3 * D.d; g.K = D.d; g.x_src = B.ra; g.x_g = g1; g.x_b = b1; g.x_store = st1;
+    g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
+    g.kdst = kc; g.vdst = vc; g.slot0 = pos0;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+
+    attn_phase<W>(D, B.q, kc, vc, B.att, M, pos0, 0, scratch);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+
+    g = GemmArgs<W>{};
+    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
+    g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+
+    const W* g2 = D.pre_ln ? L.ln2g : L.ln1g;
+    const W* b2 = D.pre_ln ? L.ln2b : L.ln1b;
+    float* st2 = D.pre_ln ? nullptr : B.xb;
+    const float* res2 = D.pre_ln ? B.rb : B.xb;
+    g = GemmArgs<W>{};
+    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.rb; g.x_g = g2; g.x_b = b2; g.x_store = st2;
+    g.w = L.wqc; g.bias = L.bqc; g.epi = EPI_STORE; g.out = B.q; g.ld = D.d;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+
+    attn_phase<W>(D, B.q, kx, vx, B.att, M, -1, P.n_src, scratch);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+
+    g = GemmArgs<W>{};
+    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.woc; g.bias = L.boc;
+    g.epi = EPI_RESID; g.out = B.rc; g.ld = D.d; g.resid = res2;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+
+    const W* g3 = D.pre_ln ? L.ln3g : L.ln2g;
+    const W* b3 = D.pre_ln ? L.ln3b : L.ln2b;
+    float* st3 = D.pre_ln ? nullptr : B.xc;
+    const float* res3 = D.pre_ln ? B.rc : B.xc;
+    g = GemmArgs<W>{};
+    g.M = M; g.N = D.f; g.K = D.d; g.x_src = B.rc; g.x_g = g3; g.x_b = b3; g.x_store = st3;
+    g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+
+    g = GemmArgs<W>{};
+    g.M = M; g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
+    g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res3;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return false;
+  }
+  return true;
+}
+
+// LM head over the final hidden rows: argmax partials (or raw logits).
+template <typename W>
+__device__ void lm_head(const KParams<W>& P, int M, unsigned char* smem, float* logits) {
+  const Dims& D = P.D;
+  const ModelW<W>& mw = *P.mw;
+  GemmArgs<W> g{};
+  g.M = M; g.N = D.V; g.K = D.d; g.x_src = P.B.ra;
+  g.x_g = D.pre_ln ? mw.dec_lnf_g : mw.dec[D.Ld - 1].ln3g;
+  g.x_b = D.pre_ln ? mw.dec_lnf_b : mw.dec[D.Ld - 1].ln3b;
+  g.w = mw.embed;
+  if (logits != nullptr) { g.epi = EPI_LOGITS; g.out = logits; g.ld = D.V; }
+  else { g.epi = EPI_ARGMAX; g.part = P.B.part; g.part_ld = D.rows; }
+  gemm_phase<W>(g, D, smem);
+}
+
+// ------------------------------------------------------------------------------------------
+// fixed-point commit (CTA 0): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
+// ------------------------------------------------------------------------------------------
+
+template <typename W>
+__device__ void commit(const KParams<W>& P, unsigned char* smem) {
+  const Dims& D = P.D;
+  const Bufs<W>& B = P.B;
+  const SmemLayout SL = smem_layout(D, sizeof(W));
+  int* ntok = reinterpret_cast<int*>(smem + SL.commit);
+  float* nprob = reinterpret_cast<float*>(ntok + D.max_tgt + 1);
+  __shared__ int s_nan;
+  volatile DecState* s = B.st;
+  const int blk = s->blk;
+  if (threadIdx.x == 0) s_nan = 0;
+  __syncthreads();
+  for (int r = threadIdx.x; r < blk; r += blockDim.x) {
+    Partial a{-INFINITY, 0x7fffffff, 0.f, 0};
+    for (int c = 0; c < (int)gridDim.x; ++c) {
+      const Partial* pp = B.part + (size_t)c * D.rows + r;
+      Partial b;
+      b.mx = __ldcg(&pp->mx);
+      b.idx = __ldcg(&pp->idx);
+      b.sum = __ldcg(&pp->sum);
+      b.nan = __ldcg(&pp->nan);
+      partial_merge(a, b);
+    }
+    ntok[r] = a.idx;
+    nprob[r] = 1.0f / a.sum;
+    if (a.nan || a.mx == -INFINITY) atomicOr(&s_nan, 1);
+  }
+  __syncthreads();
+  if (threadIdx.x != 0) return;
+
+  int* y = B.y;
+  const int i = s->i;
+  int c = 0;
+  while (c < blk && ntok[c] == y[i + c]) ++c;
+  const int stop = c == blk;
+  int eos_idx = -1;
+  for (int r = 0; r < blk; ++r)
+    if (ntok[r] == D.eos) { eos_idx = r; break; }
+  for (int r = 0; r < blk; ++r) y[i + r] = ntok[r];
+  s->k = s->k + 1;
+  const int n_it = s->n_iters + 1;
+  s->n_iters = n_it;
+  const int t = s->n_trace;
+  if (t < D.max_tgt) {
+    pd_trace_step row;
+    row.step = n_it; row.block_start = i; row.block_len = blk; row.n_converged = c;
+    row.stop = stop; row.eos_idx = eos_idx;
+    B.trace[t] = row;
+    for (int r = 0; r < blk; ++r) {
+      B.trace_tok[(size_t)t * D.max_tgt + r] = ntok[r];
+      B.trace_prob[(size_t)t * D.max_tgt + r] = nprob[r];
+    }
+    s->n_trace = t + 1;
+  }
+  if (s_nan) { s->status = PD_ENAN; s->n_y = i - 1; s->done = 1; return; }
+
+  if (stop || s->k >= blk) {                       // the block is solved
+    const bool one_pos = s->method == PD_GREEDY || s->ar_tail;
+    if (one_pos) {
+      const bool eos_ends = s->ar_tail ? true : (s->stop_at_eos != 0);
+      if (eos_ends && ntok[0] == D.eos) { s->n_y = i; s->done = 1; }
+    } else if (s->method == PD_HYBRID_GS_JACOBI && eos_idx >= 0) {
+      s->n_y = i + eos_idx;                        // through the EOS (Algorithm 3)
+      s->done = 1;
+    }
+    if (!s->done) {
+      const int ni = i + blk;
+      if (s->method == PD_HYBRID_GS_JACOBI && !s->ar_tail && ni > s->h) {
+        s->ar_tail = 1;                            // greedy tail up to max_len
+        s->b_eff = 1;
+        s->m_eff = s->max_len;
+      }
+      if (ni > s->m_eff) {
+        s->done = 1;
+        int n = s->m_eff;
+        if ((s->method == PD_JACOBI || s->method == PD_GS_JACOBI) && s->stop_at_eos) {
+          for (int p = 1; p <= s->m_eff; ++p)
+            if (y[p] == D.eos) { n = p; break; }
+        }
+        s->n_y = n;
+      } else {
+        s->i = ni;
+        const int rest = s->m_eff - ni + 1;
+        s->blk = s->b_eff < rest ? s->b_eff : rest;
+        s->k = 0;
+      }
+    }
+  }
+  // the pass budget, and a hard cap no correct schedule reaches (at most m passes for the
+  // parallel part plus max_len for a greedy tail): the loop can never run away
+  if (!s->done && ((s->max_passes > 0 && n_it >= s->max_passes) || n_it > 2 * s->max_len + 2)) {
+    s->status = PD_ENOTCONV;
+    s->n_y = s->i - 1;
+    s->done = 1;
+  }
+}
+
+template <typename W>
+__device__ void write_outputs(const KParams<W>& P) {
+  volatile DecState* s = P.B.st;
+  if (P.out_info == nullptr) return;
+  const int n_y = s->n_y;
+  for (int p = threadIdx.x; p < n_y; p += blockDim.x) P.out_y[p] = P.B.y[1 + p];
+  if (threadIdx.x == 0) {
+    P.out_info[0] = n_y;
+    P.out_info[1] = s->n_iters;
+    P.out_info[2] = s->status;
+    P.out_info[3] = s->n_trace;
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// kernels
+// ------------------------------------------------------------------------------------------
+
+template <typename W>
+__global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ int s_done, s_i, s_blk;
+  unsigned tgt = 0;
+  const Dims& D = P.D;
+  const Bufs<W>& B = P.B;
+  int* status = &B.st->status;
+
+  if (P.debug_len > 0) {
+    if (!decoder_pass<W>(P, P.debug_len, 0, B.dbg_tok, tgt, smem)) return;
+    lm_head<W>(P, P.debug_len, smem, P.logits);
+    return;
+  }
+
+  if (blockIdx.x == 0) {
+    for (int p = threadIdx.x; p <= P.init.max_len; p += blockDim.x)
+      B.y[p] = p == 0 ? D.bos : D.pad;                       // InitT: all PAD (Section 3.3)
+    if (threadIdx.x == 0) {
+      DecState s = P.init;
+      s.b_eff = s.method == PD_GREEDY ? 1 : (s.method == PD_JACOBI ? s.max_len : s.b);
+      s.m_eff = s.method == PD_HYBRID_GS_JACOBI ? s.h : s.max_len;
+      s.i = 1;
+      s.blk = s.b_eff < s.m_eff ? s.b_eff : s.m_eff;
+      s.k = 0; s.ar_tail = 0; s.n_iters = 0; s.done = 0; s.n_y = 0; s.n_trace = 0;
+      s.status = 0;
+      *B.st = s;
+    }
+  }
+  if (!grid_barrier(B.bar, tgt, status)) { if (blockIdx.x == 0) write_outputs(P); return; }
+
+  for (;;) {
+    if (threadIdx.x == 0) {
+      volatile DecState* s = B.st;
+      s_done = s->done;
+      s_i = s->i;
+      s_blk = s->blk;
+    }
+    __syncthreads();
+    if (s_done) break;
+    const int M = s_blk, pos0 = s_i - 1;
+    // row r's input is the token at position i-1+r: y_{i-1}, then the block's draft
+    // (the shift-left of Algorithm 2's appendix note)
+    if (!decoder_pass<W>(P, M, pos0, B.y + pos0, tgt, smem)) break;
+    lm_head<W>(P, M, smem, nullptr);
+    if (!grid_barrier(B.bar, tgt, status)) break;
+    if (blockIdx.x == 0) commit<W>(P, smem);
+    if (!grid_barrier(B.bar, tgt, status)) break;
+  }
+  if (blockIdx.x == 0) {
+    __syncthreads();
+    write_outputs(P);
+  }
+}
+
+template <typename W>
+__global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  unsigned tgt = 0;
+  const Dims& D = P.D;
+  const Bufs<W>& B = P.B;
+  const ModelW<W>& mw = *P.mw;
+  int* status = &B.st->status;
+  const SmemLayout SL = smem_layout(D, sizeof(W));
+  float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
+  const int n = P.n_src;
+
+  embed_phase<W>(D, mw.embed, mw.pos, D.pre_ln ? mw.enc_lne_g : nullptr,
+                 D.pre_ln ? mw.enc_lne_b : nullptr, P.enc_tok, 0, n, B.ra);
+  if (!grid_barrier(B.bar, tgt, status)) return;
+  for (int l = 0; l < D.Le; ++l) {
+    const EncLayerW<W>& L = mw.enc[l];
+    const W *g1, *b1;
+    float* st1;
+    const float* res1;
+    if (D.pre_ln) { g1 = L.ln1g; b1 = L.ln1b; st1 = nullptr; res1 = B.ra; }
+    else if (l == 0) { g1 = nullptr; b1 = nullptr; st1 = nullptr; res1 = B.ra; }
+    else { g1 = mw.enc[l - 1].ln2g; b1 = mw.enc[l - 1].ln2b; st1 = B.xa; res1 = B.xa; }
+    GemmArgs<W> g{};
+    g.M = n; g.N = 3 * D.d; g.K = D.d; g.x_src = B.ra; g.x_g = g1; g.x_b = b1; g.x_store = st1;
+    g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
+    g.kdst_f = B.k; g.vdst_f = B.v;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return;
+
+    attn_phase<float>(D, B.q, B.k, B.v, B.att, n, -1, n, scratch);
+    if (!grid_barrier(B.bar, tgt, status)) return;
+
+    g = GemmArgs<W>{};
+    g.M = n; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
+    g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return;
+
+    const W* g2 = D.pre_ln ? L.ln2g : L.ln1g;
+    const W* b2 = D.pre_ln ? L.ln2b : L.ln1b;
+    float* st2 = D.pre_ln ? nullptr : B.xb;
+    const float* res2 = D.pre_ln ? B.rb : B.xb;
+    g = GemmArgs<W>{};
+    g.M = n; g.N = D.f; g.K = D.d; g.x_src = B.rb; g.x_g = g2; g.x_b = b2; g.x_store = st2;
+    g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return;
+
+    g = GemmArgs<W>{};
+    g.M = n; g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
+    g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res2;
+    gemm_phase<W>(g, D, smem);
+    if (!grid_barrier(B.bar, tgt, status)) return;
+  }
+  // cross-attention keys and values of every decoder layer from the encoder output
+  for (int l = 0; l < D.Ld; ++l) {
+    GemmArgs<W> g{};
+    g.M = n; g.N = 2 * D.d; g.K = D.d; g.x_src = B.ra;
+    g.x_g = D.pre_ln ? mw.enc_lnf_g : mw.enc[D.Le - 1].ln2g;
+    g.x_b = D.pre_ln ? mw.enc_lnf_b : mw.enc[D.Le - 1].ln2b;
+    g.w = mw.dec[l].wkvc; g.bias = mw.dec[l].bkvc; g.epi = EPI_KVCROSS;
+    g.kdst = B.kcross + (size_t)l * D.max_src * D.d;
+    g.vdst = B.vcross + (size_t)l * D.max_src * D.d;
+    g.kv_ld = D.max_src;
+    gemm_phase<W>(g, D, smem);
+  }
+}
+
+}  // namespace pd
+
+// ============================================================================================
+// host side
+// ============================================================================================
+
+using pd::Dims;
+
+struct pd_ctx {
+  pd_config cfg;
+  Dims D;
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  int device = 0, n_sm = 0, grid = 0;
+  size_t smem = 0;
+  std::vector<void*> allocs;
+  void* wdev = nullptr;                       // device weights (tensors 256-byte aligned)
+  std::vector<size_t> woff, wbytes;           // per tensor, blob order
+  size_t blob_bytes = 0;
+  void* mw_dev = nullptr;                     // ModelW<W> table on the device
+  pd::Bufs<float> bf{};
+  pd::Bufs<__nv_bfloat16> bb{};
+  int32_t* d_out_y = nullptr;
+  int32_t* d_out_info = nullptr;
+  int n_src = 0;
+  bool encoded = false;
+  int64_t launches = 0;
+  std::string err;
+};
+
+namespace {
+
+pd_status fail(pd_ctx* c, pd_status s, const std::string& msg) {
+  if (c) c->err = msg;
+  return s;
+}
+
+#define PD_CUDA(ctx, call)                                                             \
+  do {                                                                                 \
+    cudaError_t e_ = (call);                                                           \
+    if (e_ != cudaSuccess)                                                             \
+      return fail(ctx, PD_ECUDA, std::string(#call ": ") + cudaGetErrorString(e_));    \
+  } while (0)
+
+size_t wsize(const pd_config& c) { return c.dtype == PD_DTYPE_BF16 ? 2 : 4; }
+
+bool valid_config(const pd_config* c, std::string* why) {
+  auto bad = [&](const char* m) { if (why) *why = m; return false; };
+  if (!c) return bad("cfg is NULL");
+  if (c->dtype != PD_DTYPE_F32 && c->dtype != PD_DTYPE_BF16) return bad("dtype");
+  if (c->d_model <= 0 || c->d_model % 256) return bad("d_model must be a positive multiple of 256");
+  if (c->d_ff <= 0 || c->d_ff % 256) return bad("d_ff must be a positive multiple of 256");
+  if (c->n_heads <= 0 || c->d_model % c->n_heads) return bad("n_heads must divide d_model");
+  const int dh = c->d_model / c->n_heads;
+  if (dh != 32 && dh != 64 && dh != 128) return bad("d_model / n_heads must be 32, 64 or 128");
+  if (c->n_enc_layers < 1 || c->n_enc_layers > pd::kMaxLayers) return bad("n_enc_layers");
+  if (c->n_dec_layers < 1 || c->n_dec_layers > pd::kMaxLayers) return bad("n_dec_layers");
+  if (c->vocab < 4) return bad("vocab");
+  if (c->activation < 0 || c->activation > 2) return bad("activation");
+  if (c->learned_pos && c->max_pos < 1) return bad("max_pos");
+  if (c->max_src_len < 1 || c->max_tgt_len < 1 || c->max_src_len > 4096 || c->max_tgt_len > 4096)
+    return bad("max_src_len / max_tgt_len must be in [1, 4096]");
+  for (int id : {c->pad_id, c->eos_id, c->bos_id})
+    if (id < 0 || id >= c->vocab) return bad("special ids must be in [0, vocab)");
+  if (!(c->ln_eps >= 0.f)) return bad("ln_eps");
+  return true;
+}
+
+// Tensor sizes (elements) in blob order; the same order fills the pointer table.
+template <typename W>
+std::vector<std::pair<const W**, size_t>> layout(pd::ModelW<W>& mw, const pd_config& c) {
+  const size_t d = c.d_model, f = c.d_ff, V = c.vocab;
+  std::vector<std::pair<const W**, size_t>> t;
+  t.push_back({&mw.embed, V * d});
+  if (c.learned_pos) t.push_back({&mw.pos, (size_t)c.max_pos * d});
+  if (c.pre_ln) {
+    t.push_back({&mw.enc_lne_g, d}); t.push_back({&mw.enc_lne_b, d});
+    t.push_back({&mw.dec_lne_g, d}); t.push_back({&mw.dec_lne_b, d});
+    t.push_back({&mw.enc_lnf_g, d}); t.push_back({&mw.enc_lnf_b, d});
+    t.push_back({&mw.dec_lnf_g, d}); t.push_back({&mw.dec_lnf_b, d});
+  }
+  for (int l = 0; l < c.n_enc_layers; ++l) {
+    auto& L = mw.enc[l];
+    t.push_back({&L.wqkv, 3 * d * d}); t.push_back({&L.bqkv, 3 * d});
+    t.push_back({&L.wo, d * d}); t.push_back({&L.bo, d});
+    t.push_back({&L.ln1g, d}); t.push_back({&L.ln1b, d});
+    t.push_back({&L.w1, f * d}); t.push_back({&L.b1, f});
+    t.push_back({&L.w2, d * f}); t.push_back({&L.b2, d});
+    t.push_back({&L.ln2g, d}); t.push_back({&L.ln2b, d});
+  }
+  for (int l = 0; l < c.n_dec_layers; ++l) {
+    auto& L = mw.dec[l];
+    t.push_back({&L.wqkv, 3 * d * d}); t.push_back({&L.bqkv, 3 * d});
+    t.push_back({&L.wo, d * d}); t.push_back({&L.bo, d});
+    t.push_back({&L.ln1g, d}); t.push_back({&L.ln1b, d});
+    t.push_back({&L.wqc, d * d}); t.push_back({&L.bqc, d});
+    t.push_back({&L.wkvc, 2 * d * d}); t.push_back({&L.bkvc, 2 * d});
+    t.push_back({&L.woc, d * d}); t.push_back({&L.boc, d});
+    t.push_back({&L.ln2g, d}); t.push_back({&L.ln2b, d});
+    t.push_back({&L.w1, f * d}); t.push_back({&L.b1, f});
+    t.push_back({&L.w2, d * f}); t.push_back({&L.b2, d});
+    t.push_back({&L.ln3g, d}); t.push_back({&L.ln3b, d});
+  }
+  return t;
+}
+
+size_t blob_elems(const pd_config& c) {
+  pd::ModelW<float> mw{};
+  size_t n = 0;
+  for (auto& e : layout<float>(mw, c)) n += e.second;
+  return n;
+}
+
+template <typename W>
+pd::Bufs<W>& bufs(pd_ctx* c);
+template <> pd::Bufs<float>& bufs<float>(pd_ctx* c) { return c->bf; }
+template <> pd::Bufs<__nv_bfloat16>& bufs<__nv_bfloat16>(pd_ctx* c) { return c->bb; }
+
+template <typename T>
+pd_status dalloc(pd_ctx* c, T** p, size_t count) {
+  void* q = nullptr;
+  cudaError_t e = cudaMalloc(&q, count * sizeof(T) > 0 ? count * sizeof(T) : 16);
+  if (e != cudaSuccess) return fail(c, PD_ENOMEM, std::string("cudaMalloc: ") + cudaGetErrorString(e));
+  c->allocs.push_back(q);
+  *p = static_cast<T*>(q);
+  return PD_OK;
+}
+
+#define PD_TRY(expr)               \
+  do {                             \
+    pd_status s_ = (expr);         \
+    if (s_ != PD_OK) return s_;    \
+  } while (0)
+
+template <typename W>
+pd_status create_impl(pd_ctx* c, const void* weights) {
+  const pd_config& cfg = c->cfg;
+  Dims& D = c->D;
+  // weights: each tensor at a 256-byte aligned offset of one allocation
+  pd::ModelW<W> mw{};
+  auto lay = layout<W>(mw, cfg);
+  size_t off = 0;
+  for (auto& e : lay) {
+    c->woff.push_back(off);
+    c->wbytes.push_back(e.second * sizeof(W));
+    off += (e.second * sizeof(W) + 255) / 256 * 256;
+  }
+  unsigned char* wdev = nullptr;
+  PD_TRY(dalloc(c, &wdev, off));
+  c->wdev = wdev;
+  const unsigned char* src = static_cast<const unsigned char*>(weights);
+  size_t soff = 0;
+  for (size_t k = 0; k < lay.size(); ++k) {
+    *lay[k].first = reinterpret_cast<const W*>(wdev + c->woff[k]);
+    PD_CUDA(c, cudaMemcpy(wdev + c->woff[k], src + soff, c->wbytes[k], cudaMemcpyHostToDevice));
+    soff += c->wbytes[k];
+  }
+  pd::ModelW<W>* mwd = nullptr;
+  PD_TRY(dalloc(c, &mwd, 1));
+  PD_CUDA(c, cudaMemcpy(mwd, &mw, sizeof(mw), cudaMemcpyHostToDevice));
+  c->mw_dev = mwd;
+
+  pd::Bufs<W>& B = bufs<W>(c);
+  const size_t R = D.rows, d = D.d;
+  PD_TRY(dalloc(c, &B.ra, R * d)); PD_TRY(dalloc(c, &B.rb, R * d)); PD_TRY(dalloc(c, &B.rc, R * d));
+  PD_TRY(dalloc(c, &B.xa, R * d)); PD_TRY(dalloc(c, &B.xb, R * d)); PD_TRY(dalloc(c, &B.xc, R * d));
+  PD_TRY(dalloc(c, &B.q, R * d)); PD_TRY(dalloc(c, &B.k, R * d)); PD_TRY(dalloc(c, &B.v, R * d));
+  PD_TRY(dalloc(c, &B.att, R * d));
+  PD_TRY(dalloc(c, &B.ffh, R * (size_t)D.f));
+  PD_TRY(dalloc(c, &B.kself, (size_t)D.Ld * D.max_tgt * d));
+  PD_TRY(dalloc(c, &B.vself, (size_t)D.Ld * D.max_tgt * d));
+  PD_TRY(dalloc(c, &B.kcross, (size_t)D.Ld * D.max_src * d));
+  PD_TRY(dalloc(c, &B.vcross, (size_t)D.Ld * D.max_src * d));
+  PD_TRY(dalloc(c, &B.part, (size_t)c->grid * R));
+  PD_TRY(dalloc(c, &B.y, (size_t)D.max_tgt + 1));
+  PD_TRY(dalloc(c, &B.st, 1));
+  PD_TRY(dalloc(c, &B.trace, (size_t)D.max_tgt));
+  PD_TRY(dalloc(c, &B.trace_tok, (size_t)D.max_tgt * D.max_tgt));
+  PD_TRY(dalloc(c, &B.trace_prob, (size_t)D.max_tgt * D.max_tgt));
+  PD_TRY(dalloc(c, &B.bar, 2));
+  PD_TRY(dalloc(c, &B.src, (size_t)D.max_src));
+  PD_TRY(dalloc(c, &B.dbg_tok, (size_t)D.max_tgt));
+  PD_TRY(dalloc(c, &c->d_out_y, (size_t)D.max_tgt));
+  PD_TRY(dalloc(c, &c->d_out_info, 4));
+  PD_CUDA(c, cudaMemset(B.st, 0, sizeof(pd::DecState)));
+  PD_CUDA(c, cudaMemset(B.bar, 0, 2 * sizeof(unsigned)));
+
+  c->smem = pd::smem_layout(D, sizeof(W)).total;
+  PD_CUDA(c, cudaFuncSetAttribute(pd::decode_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)c->smem));
+  PD_CUDA(c, cudaFuncSetAttribute(pd::encode_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)c->smem));
+  int nb1 = 0, nb2 = 0;
+  PD_CUDA(c, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb1, pd::decode_kernel<W>, pd::kThreads,
+                                                           c->smem));
+  PD_CUDA(c, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb2, pd::encode_kernel<W>, pd::kThreads,
+                                                           c->smem));
+  if (nb1 < 1 || nb2 < 1) return fail(c, PD_EINVAL, "kernel does not fit on an SM (shared memory)");
+  return PD_OK;
+}
+
+template <typename W>
+pd::KParams<W> base_params(pd_ctx* c) {
+  pd::KParams<W> P{};
+  P.D = c->D;
+  P.mw = static_cast<const pd::ModelW<W>*>(c->mw_dev);
+  P.B = bufs<W>(c);
+  P.n_src = c->n_src;
+  return P;
+}
+
+template <typename W>
+pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P) {
+  PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).bar, 0, 2 * sizeof(unsigned), c->stream));
+  if (encode) PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).st, 0, sizeof(pd::DecState), c->stream));
+  void* args[] = {&P};
+  const void* fn = encode ? (const void*)pd::encode_kernel<W> : (const void*)pd::decode_kernel<W>;
+  PD_CUDA(c, cudaLaunchCooperativeKernel(fn, dim3(c->grid), dim3(pd::kThreads), args, c->smem,
+                                         c->stream));
+  c->launches += 1;
+  return PD_OK;
+}
+
+template <typename W>
+pd_status encode_impl(pd_ctx* c, const int32_t* d_src, int n) {
+  pd::KParams<W> P = base_params<W>(c);
+  P.n_src = n;
+  P.enc_tok = d_src;
+  PD_TRY(launch<W>(c, true, P));
+  c->n_src = n;
+  c->encoded = true;
+  return PD_OK;
+}
+
+template <typename W>
+pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int32_t* d_y, int32_t* d_info) {
+  pd::KParams<W> P = base_params<W>(c);
+  P.init = pd::DecState{};
+  P.init.method = p->method;
+  P.init.b = p->b;
+  P.init.max_len = p->max_len;
+  P.init.h = (p->h <= 0 || p->h > p->max_len) ? p->max_len : p->h;
+  P.init.stop_at_eos = p->stop_at_eos;
+  P.init.max_passes = p->max_passes;
+  P.out_y = d_y;
+  P.out_info = d_info;
+  return launch<W>(c, false, P);
+}
+
+template <typename W>
+pd_status debug_impl(pd_ctx* c, int len, float* d_logits) {
+  pd::KParams<W> P = base_params<W>(c);
+  P.debug_len = len;
+  P.logits = d_logits;
+  return launch<W>(c, false, P);
+}
+
+pd_status check_params(pd_ctx* c, const pd_decode_params* p) {
+  if (!p) return fail(c, PD_EINVAL, "params is NULL");
+  if (p->method < PD_GREEDY || p->method > PD_HYBRID_GS_JACOBI) return fail(c, PD_EINVAL, "method");
+  if (p->max_len < 1 || p->max_len > c->cfg.max_tgt_len)
+    return fail(c, PD_EINVAL, "max_len must be in [1, max_tgt_len]");
+  if ((p->method == PD_GS_JACOBI || p->method == PD_HYBRID_GS_JACOBI) && p->b < 1)
+    return fail(c, PD_EINVAL, "b must be >= 1");
+  if (p->max_passes < 0) return fail(c, PD_EINVAL, "max_passes must be >= 0");
+  if (c->cfg.learned_pos && p->max_len > c->cfg.max_pos)
+    return fail(c, PD_EINVAL, "max_len exceeds the learned position table");
+  if (!c->encoded) return fail(c, PD_ESTATE, "pd_decode before pd_encode");
+  return PD_OK;
+}
+
+}  // namespace
+
+// ============================================================================================
+// C ABI
+// ============================================================================================
+
+extern "C" {
+
+size_t pd_weights_nbytes(const pd_config* cfg) {
+  if (!valid_config(cfg, nullptr)) return 0;
+  return blob_elems(*cfg) * wsize(*cfg);
+}
+
+pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, void* stream,
+                    pd_ctx** out) {
+  if (!out) return PD_EINVAL;
+  *out = nullptr;
+  std::string why;
+  if (!valid_config(cfg, &why)) return PD_EINVAL;
+  if (!weights || nbytes != pd_weights_nbytes(cfg)) return PD_EINVAL;
+  pd_ctx* c = new pd_ctx();
+  c->cfg = *cfg;
+  Dims& D = c->D;
+  D.d = cfg->d_model; D.H = cfg->n_heads; D.dh = cfg->d_model / cfg->n_heads; D.f = cfg->d_ff;
+  D.Le = cfg->n_enc_layers; D.Ld = cfg->n_dec_layers; D.V = cfg->vocab;
+  D.act = cfg->activation; D.pre_ln = cfg->pre_ln ? 1 : 0; D.learned_pos = cfg->learned_pos ? 1 : 0;
+  D.max_pos = cfg->learned_pos ? cfg->max_pos : 1;
+  D.pad = cfg->pad_id; D.eos = cfg->eos_id; D.bos = cfg->bos_id;
+  D.eps = cfg->ln_eps; D.emb_scale = sqrtf((float)cfg->d_model);
+  D.max_src = cfg->max_src_len; D.max_tgt = cfg->max_tgt_len;
+  D.rows = D.max_src > D.max_tgt ? D.max_src : D.max_tgt;
+  c->blob_bytes = nbytes;
+  pd_status s = PD_OK;
+  cudaError_t e = cudaGetDevice(&c->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);
+  int coop = 0;
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, c->device);
+  if (e != cudaSuccess || !coop) {
+    pd_destroy(c);
+    return PD_ECUDA;
+  }
+  c->grid = c->n_sm;
+  if (stream) {
+    c->stream = static_cast<cudaStream_t>(stream);
+  } else {
+    if (cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking) != cudaSuccess) {
+      pd_destroy(c);
+      return PD_ECUDA;
+    }
+    c->own_stream = true;
+  }
+  s = cfg->dtype == PD_DTYPE_BF16 ? create_impl<__nv_bfloat16>(c, weights)
+                                  : create_impl<float>(c, weights);
+  if (s != PD_OK) {
+    pd_destroy(c);
+    return s;
+  }
+  *out = c;
+  return PD_OK;
+}
+
+pd_status pd_export_weights(pd_ctx* c, void* dst, size_t nbytes) {
+  if (!c) return PD_EINVAL;
+  if (!dst || nbytes != c->blob_bytes) return fail(c, PD_EINVAL, "dst size must equal the blob size");
+  unsigned char* o = static_cast<unsigned char*>(dst);
+  size_t off = 0;
+  for (size_t k = 0; k < c->woff.size(); ++k) {
+    PD_CUDA(c, cudaMemcpy(o + off, static_cast<unsigned char*>(c->wdev) + c->woff[k], c->wbytes[k],
+                          cudaMemcpyDeviceToHost));
+    off += c->wbytes[k];
+  }
+  return PD_OK;
+}
+
+pd_status pd_encode_device(pd_ctx* c, const int32_t* d_src, int n_src) {
+  if (!c) return PD_EINVAL;
+  if (!d_src || n_src < 1 || n_src > c->cfg.max_src_len)
+    return fail(c, PD_EINVAL, "n_src must be in [1, max_src_len]");
+  if (c->cfg.learned_pos && n_src > c->cfg.max_pos)
+    return fail(c, PD_EINVAL, "n_src exceeds the learned position table");
+  return c->cfg.dtype == PD_DTYPE_BF16 ? encode_impl<__nv_bfloat16>(c, d_src, n_src)
+                                       : encode_impl<float>(c, d_src, n_src);
+}
+
+pd_status pd_encode(pd_ctx* c, const int32_t* src, int n_src) {
+  if (!c) return PD_EINVAL;
+  if (!src || n_src < 1 || n_src > c->cfg.max_src_len)
+    return fail(c, PD_EINVAL, "n_src must be in [1, max_src_len]");
+  for (int k = 0; k < n_src; ++k)
+    if (src[k] < 0 || src[k] >= c->cfg.vocab) return fail(c, PD_EINVAL, "source id out of range");
+  int32_t* dsrc = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.src : c->bf.src;
+  PD_CUDA(c, cudaMemcpyAsync(dsrc, src, n_src * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  PD_TRY(pd_encode_device(c, dsrc, n_src));
+  PD_CUDA(c, cudaStreamSynchronize(c->stream));
+  int st = 0;
+  pd::DecState* dst = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.st : c->bf.st;
+  PD_CUDA(c, cudaMemcpy(&st, &dst->status, sizeof(int), cudaMemcpyDeviceToHost));
+  if (st != 0) {
+    c->encoded = false;
+    return fail(c, (pd_status)st, "encoder kernel reported a failure");
+  }
+  return PD_OK;
+}
+
+pd_status pd_decode_device(pd_ctx* c, const pd_decode_params* p, int32_t* d_y, int32_t* d_info) {
+  if (!c) return PD_EINVAL;
+  PD_TRY(check_params(c, p));
+  if (!d_y || !d_info) return fail(c, PD_EINVAL, "d_y and d_info are required");
+  return c->cfg.dtype == PD_DTYPE_BF16 ? decode_impl<__nv_bfloat16>(c, p, d_y, d_info)
+                                       : decode_impl<float>(c, p, d_y, d_info);
+}
+
+pd_status pd_decode(pd_ctx* c, const pd_decode_params* p, int32_t* y, int* n_y, int* n_iters,
+                    pd_trace_step* trace, int32_t* trace_tokens, float* trace_probs, int trace_cap,
+                    int* n_trace) {
+  if (!c) return PD_EINVAL;
+  PD_TRY(check_params(c, p));
+  if (!y || !n_y || !n_iters) return fail(c, PD_EINVAL, "y, n_y and n_iters are required");
+  if (trace && (trace_cap < 0 || !n_trace)) return fail(c, PD_EINVAL, "trace needs trace_cap and n_trace");
+  PD_TRY(pd_decode_device(c, p, c->d_out_y, c->d_out_info));
+  int32_t info[4];
+  PD_CUDA(c, cudaMemcpyAsync(info, c->d_out_info, sizeof(info), cudaMemcpyDeviceToHost, c->stream));
+  PD_CUDA(c, cudaStreamSynchronize(c->stream));
+  const int ny = info[0] < 0 ? 0 : (info[0] > p->max_len ? p->max_len : info[0]);
+  if (ny > 0)
+    PD_CUDA(c, cudaMemcpy(y, c->d_out_y, ny * sizeof(int32_t), cudaMemcpyDeviceToHost));
+  *n_y = ny;
+  *n_iters = info[1];
+  if (trace) {
+    const int D_tgt = c->cfg.max_tgt_len;
+    const int nt = info[3] < trace_cap ? info[3] : trace_cap;
+    pd_trace_step* dtr = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.trace : c->bf.trace;
+    int* dtt = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.trace_tok : c->bf.trace_tok;
+    float* dtp = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.trace_prob : c->bf.trace_prob;
+    if (nt > 0) {
+      PD_CUDA(c, cudaMemcpy(trace, dtr, nt * sizeof(pd_trace_step), cudaMemcpyDeviceToHost));
+      if (trace_tokens || trace_probs) {
+        // device rows have stride max_tgt_len; the caller's rows have stride max_len
+        PD_CUDA(c, cudaMemcpy2D(trace_tokens ? (void*)trace_tokens : (void*)trace_probs,
+                                p->max_len * sizeof(int32_t), trace_tokens ? (void*)dtt : (void*)dtp,
+                                D_tgt * sizeof(int32_t), p->max_len * sizeof(int32_t), nt,
+                                cudaMemcpyDeviceToHost));
+        if (trace_tokens && trace_probs)
+          PD_CUDA(c, cudaMemcpy2D(trace_probs, p->max_len * sizeof(float), dtp, D_tgt * sizeof(float),
+                                  p->max_len * sizeof(float), nt, cudaMemcpyDeviceToHost));
+      }
+    }
+    *n_trace = nt;
+  }
+  const int st = info[2];
+  if (st != 0) return fail(c, (pd_status)st, st == PD_ENOTCONV ? "pass budget exhausted"
+                                               : st == PD_ENAN ? "NaN in the logits"
+                                               : "decode kernel reported a failure");
+  return PD_OK;
+}
+
+pd_status pd_debug_logits(pd_ctx* c, const int32_t* y_in, int len, float* logits) {
+  if (!c) return PD_EINVAL;
+  if (!y_in || !logits || len < 1 || len > c->cfg.max_tgt_len)
+    return fail(c, PD_EINVAL, "len must be in [1, max_tgt_len]");
+  if (c->cfg.learned_pos && len > c->cfg.max_pos) return fail(c, PD_EINVAL, "len exceeds max_pos");
+  for (int k = 0; k < len; ++k)
+    if (y_in[k] < 0 || y_in[k] >= c->cfg.vocab) return fail(c, PD_EINVAL, "token id out of range");
+  if (!c->encoded) return fail(c, PD_ESTATE, "pd_debug_logits before pd_encode");
+  int* dtok = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.dbg_tok : c->bf.dbg_tok;
+  PD_CUDA(c, cudaMemcpyAsync(dtok, y_in, len * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  float* dl = nullptr;
+  const size_t nb = (size_t)len * c->cfg.vocab * sizeof(float);
+  PD_CUDA(c, cudaMalloc(&dl, nb));
+  pd_status s = c->cfg.dtype == PD_DTYPE_BF16 ? debug_impl<__nv_bfloat16>(c, len, dl)
+                                               : debug_impl<float>(c, len, dl);
+  cudaError_t e = s == PD_OK ? cudaStreamSynchronize(c->stream) : cudaSuccess;
+  if (s == PD_OK && e == cudaSuccess) e = cudaMemcpy(logits, dl, nb, cudaMemcpyDeviceToHost);
+  cudaFree(dl);
+  if (s != PD_OK) return s;
+  if (e != cudaSuccess) return fail(c, PD_ECUDA, std::string("debug logits: ") + cudaGetErrorString(e));
+  return PD_OK;
+}
+
+void* pd_stream(pd_ctx* c) { return c ? (void*)c->stream : nullptr; }
+
+int64_t pd_launch_count(const pd_ctx* c) { return c ? c->launches : 0; }
+
+const char* pd_last_error(const pd_ctx* c) { return c ? c->err.c_str() : "context is NULL"; }
+
+void pd_destroy(pd_ctx* c) {
+  if (!c) return;
+  if (c->stream) cudaStreamSynchronize(c->stream);
+  for (void* p : c->allocs) cudaFree(p);
+  if (c->own_stream && c->stream) cudaStreamDestroy(c->stream);
+  delete c;
+}
+
+}  // extern "C"
