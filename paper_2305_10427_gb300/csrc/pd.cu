@@ -44,7 +44,7 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   const int kmax = D.d > D.f ? D.d : D.f;
   L.xs = 0;
   L.part = L.xs + ((size_t)kMTile * kmax * wsize + 15) / 16 * 16;
-  L.scratch = L.part + (size_t)kWarps * kMTile * sizeof(Partial);
+  L.scratch = L.part + (size_t)kWarps * 32 * sizeof(Partial);
   L.commit = L.scratch + (size_t)kWarps * (128 + D.rows + 4) * sizeof(float);
   L.total = L.commit + (size_t)(D.max_tgt + 1) * 2 * sizeof(int) + 64;
   return L;
@@ -55,6 +55,32 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
 // ------------------------------------------------------------------------------------------
 
 template <typename W>
+__device__ __forceinline__ EmbedTabs<W> embed_tabs(const KParams<W>& P) {
+  const ModelW<W>& mw = *P.mw;
+  return EmbedTabs<W>{mw.embed, P.D.learned_pos ? mw.pos : nullptr,
+                      P.D.learned_pos ? nullptr : P.B.pos_tab};
+}
+
+// Every weight row this CTA will read in one decoder pass, requested from L2 in phase order
+// at the start of the pass: HBM streams the pass's weights while the (latency-bound) chain
+// of phases runs, and each phase then finds its rows in L2.
+template <typename W>
+__device__ void prefetch_pass(const KParams<W>& P) {
+  const Dims& D = P.D;
+  const ModelW<W>& mw = *P.mw;
+  for (int l = 0; l < D.Ld; ++l) {
+    const DecLayerW<W>& L = mw.dec[l];
+    prefetch_gemm_weights(L.wqkv, 3 * D.d, D.d);
+    prefetch_gemm_weights(L.wo, D.d, D.d);
+    prefetch_gemm_weights(L.wqc, D.d, D.d);
+    prefetch_gemm_weights(L.woc, D.d, D.d);
+    prefetch_gemm_weights(L.w1, D.f, D.d);
+    prefetch_gemm_weights(L.w2, D.d, D.f);
+  }
+  prefetch_gemm_weights(mw.embed, D.V, D.d);
+}
+
+template <typename W>
 __device__ bool decoder_pass(const KParams<W>& P, int M, int pos0, const int* tok,
                              unsigned& tgt, unsigned char* smem) {
   const Dims& D = P.D;
@@ -63,10 +89,8 @@ __device__ bool decoder_pass(const KParams<W>& P, int M, int pos0, const int* to
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
-
-  embed_phase<W>(D, mw.embed, mw.pos, D.pre_ln ? mw.dec_lne_g : nullptr,
-                 D.pre_ln ? mw.dec_lne_b : nullptr, tok, pos0, M, B.ra);
-  if (!grid_barrier(B.bar, tgt, status)) return false;
+  const EmbedTabs<W> T = embed_tabs(P);
+  const bool pre = D.pre_ln != 0;
 
   for (int l = 0; l < D.Ld; ++l) {
     const DecLayerW<W>& L = mw.dec[l];
@@ -74,21 +98,24 @@ __device__ bool decoder_pass(const KParams<W>& P, int M, int pos0, const int* to
     W* vc = B.vself + (size_t)l * D.max_tgt * D.d;
     W* kx = B.kcross + (size_t)l * D.max_src * D.d;
     W* vx = B.vcross + (size_t)l * D.max_src * D.d;
-    // sublayer inputs: pre-LN normalises with the sublayer's own LN and keeps the raw
-    // residual; post-LN normalises with the previous sublayer's LN and that normalised row
-    // is the residual (the first sublayer takes the embedding as is).
-    const W *g1, *b1;
-    float *st1;
-    const float* res1;
-    if (D.pre_ln) { g1 = L.ln1g; b1 = L.ln1b; st1 = nullptr; res1 = B.ra; }
-    else if (l == 0) { g1 = nullptr; b1 = nullptr; st1 = nullptr; res1 = B.ra; }
-    else { g1 = mw.dec[l - 1].ln3g; b1 = mw.dec[l - 1].ln3b; st1 = B.xa; res1 = B.xa; }
 
+    // self-attention sublayer input.  Pre-LN: x = LN1(r), residual r.  Post-LN: x = the
+    // previous sublayer's LN of its output, which is also the residual; layer 0 takes the
+    // embedding as is.  The embedding is computed in this GEMM's prologue.
     GemmArgs<W> g{};
-    g.M = M; g.N = 3 * D.d; g.K = D.d; g.x_src = B.ra; g.x_g = g1; g.x_b = b1; g.x_store = st1;
+    g.M = M; g.N = 3 * D.d; g.K = D.d;
+    if (l == 0) {
+      g.emb_tok = tok; g.emb_pos0 = pos0; g.x_store = B.ra;
+      if (pre) { g.ln_a_g = mw.dec_lne_g; g.ln_a_b = mw.dec_lne_b; g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
+    } else {
+      g.x_src = B.ra;
+      if (pre) { g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
+      else { g.ln_a_g = mw.dec[l - 1].ln3g; g.ln_a_b = mw.dec[l - 1].ln3b; g.x_store = B.xa; }
+    }
+    const float* res1 = (pre || l == 0) ? B.ra : B.xa;
     g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
     g.kdst = kc; g.vdst = vc; g.slot0 = pos0;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return false;
 
     attn_phase<W>(D, B.q, kc, vc, B.att, M, pos0, 0, scratch);
@@ -97,17 +124,16 @@ __device__ bool decoder_pass(const KParams<W>& P, int M, int pos0, const int* to
     g = GemmArgs<W>{};
     g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
     g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return false;
 
-    const W* g2 = D.pre_ln ? L.ln2g : L.ln1g;
-    const W* b2 = D.pre_ln ? L.ln2b : L.ln1b;
-    float* st2 = D.pre_ln ? nullptr : B.xb;
-    const float* res2 = D.pre_ln ? B.rb : B.xb;
     g = GemmArgs<W>{};
-    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.rb; g.x_g = g2; g.x_b = b2; g.x_store = st2;
+    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.rb;
+    if (pre) { g.ln_b_g = L.ln2g; g.ln_b_b = L.ln2b; }
+    else { g.ln_a_g = L.ln1g; g.ln_a_b = L.ln1b; g.x_store = B.xb; }
+    const float* res2 = pre ? B.rb : B.xb;
     g.w = L.wqc; g.bias = L.bqc; g.epi = EPI_STORE; g.out = B.q; g.ld = D.d;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return false;
 
     attn_phase<W>(D, B.q, kx, vx, B.att, M, -1, P.n_src, scratch);
@@ -116,23 +142,22 @@ __device__ bool decoder_pass(const KParams<W>& P, int M, int pos0, const int* to
     g = GemmArgs<W>{};
     g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.woc; g.bias = L.boc;
     g.epi = EPI_RESID; g.out = B.rc; g.ld = D.d; g.resid = res2;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return false;
 
-    const W* g3 = D.pre_ln ? L.ln3g : L.ln2g;
-    const W* b3 = D.pre_ln ? L.ln3b : L.ln2b;
-    float* st3 = D.pre_ln ? nullptr : B.xc;
-    const float* res3 = D.pre_ln ? B.rc : B.xc;
     g = GemmArgs<W>{};
-    g.M = M; g.N = D.f; g.K = D.d; g.x_src = B.rc; g.x_g = g3; g.x_b = b3; g.x_store = st3;
+    g.M = M; g.N = D.f; g.K = D.d; g.x_src = B.rc;
+    if (pre) { g.ln_b_g = L.ln3g; g.ln_b_b = L.ln3b; }
+    else { g.ln_a_g = L.ln2g; g.ln_a_b = L.ln2b; g.x_store = B.xc; }
+    const float* res3 = pre ? B.rc : B.xc;
     g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return false;
 
     g = GemmArgs<W>{};
     g.M = M; g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
     g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res3;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return false;
   }
   return true;
@@ -145,20 +170,29 @@ __device__ void lm_head(const KParams<W>& P, int M, unsigned char* smem, float* 
   const ModelW<W>& mw = *P.mw;
   GemmArgs<W> g{};
   g.M = M; g.N = D.V; g.K = D.d; g.x_src = P.B.ra;
-  g.x_g = D.pre_ln ? mw.dec_lnf_g : mw.dec[D.Ld - 1].ln3g;
-  g.x_b = D.pre_ln ? mw.dec_lnf_b : mw.dec[D.Ld - 1].ln3b;
+  g.ln_b_g = D.pre_ln ? mw.dec_lnf_g : mw.dec[D.Ld - 1].ln3g;
+  g.ln_b_b = D.pre_ln ? mw.dec_lnf_b : mw.dec[D.Ld - 1].ln3b;
   g.w = mw.embed;
   if (logits != nullptr) { g.epi = EPI_LOGITS; g.out = logits; g.ld = D.V; }
   else { g.epi = EPI_ARGMAX; g.part = P.B.part; g.part_ld = D.rows; }
-  gemm_phase<W>(g, D, smem);
+  gemm_phase<W>(g, embed_tabs(P), D, smem);
 }
 
 // ------------------------------------------------------------------------------------------
-// fixed-point commit (CTA 0): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
+// fixed-point commit (one CTA): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
 // ------------------------------------------------------------------------------------------
 
+__device__ __forceinline__ Partial shfl_partial(const Partial& a, int o) {
+  Partial b;
+  b.mx = __shfl_xor_sync(0xffffffffu, a.mx, o);
+  b.idx = __shfl_xor_sync(0xffffffffu, a.idx, o);
+  b.sum = __shfl_xor_sync(0xffffffffu, a.sum, o);
+  b.nan = __shfl_xor_sync(0xffffffffu, a.nan, o);
+  return b;
+}
+
 template <typename W>
-__device__ void commit(const KParams<W>& P, unsigned char* smem) {
+__device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
   const SmemLayout SL = smem_layout(D, sizeof(W));
@@ -167,22 +201,24 @@ __device__ void commit(const KParams<W>& P, unsigned char* smem) {
   __shared__ int s_nan;
   volatile DecState* s = B.st;
   const int blk = s->blk;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) s_nan = 0;
   __syncthreads();
-  for (int r = threadIdx.x; r < blk; r += blockDim.x) {
+  // per row: the CTA partials merged lane-wise in ascending CTA order, then by a fixed
+  // butterfly (the merge is symmetric, so every lane ends with the same result)
+  for (int r = warp; r < blk; r += kWarps) {
     Partial a{-INFINITY, 0x7fffffff, 0.f, 0};
-    for (int c = 0; c < (int)gridDim.x; ++c) {
-      const Partial* pp = B.part + (size_t)c * D.rows + r;
-      Partial b;
-      b.mx = __ldcg(&pp->mx);
-      b.idx = __ldcg(&pp->idx);
-      b.sum = __ldcg(&pp->sum);
-      b.nan = __ldcg(&pp->nan);
+    for (int c = lane; c < (int)gridDim.x; c += 32) partial_merge(a, B.part[(size_t)c * D.rows + r]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const Partial b = shfl_partial(a, o);
       partial_merge(a, b);
     }
-    ntok[r] = a.idx;
-    nprob[r] = 1.0f / a.sum;
-    if (a.nan || a.mx == -INFINITY) atomicOr(&s_nan, 1);
+    if (lane == 0) {
+      ntok[r] = a.idx;
+      nprob[r] = 1.0f / a.sum;
+      if (a.nan || a.mx == -INFINITY) atomicOr(&s_nan, 1);
+    }
   }
   __syncthreads();
   if (threadIdx.x != 0) return;
@@ -313,13 +349,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
     __syncthreads();
     if (s_done) break;
     const int M = s_blk, pos0 = s_i - 1;
+    prefetch_pass<W>(P);
     // row r's input is the token at position i-1+r: y_{i-1}, then the block's draft
     // (the shift-left of Algorithm 2's appendix note)
     if (!decoder_pass<W>(P, M, pos0, B.y + pos0, tgt, smem)) break;
     lm_head<W>(P, M, smem, nullptr);
-    if (!grid_barrier(B.bar, tgt, status)) break;
-    if (blockIdx.x == 0) commit<W>(P, smem);
-    if (!grid_barrier(B.bar, tgt, status)) break;
+    // the last CTA to finish its LM-head columns merges the argmax partials and commits
+    if (!grid_barrier_last(B.bar, tgt, status, [&] { commit<W>(P, smem); })) break;
   }
   if (blockIdx.x == 0) {
     __syncthreads();
@@ -337,24 +373,35 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
+  const EmbedTabs<W> T = embed_tabs(P);
+  const bool pre = D.pre_ln != 0;
   const int n = P.n_src;
 
-  embed_phase<W>(D, mw.embed, mw.pos, D.pre_ln ? mw.enc_lne_g : nullptr,
-                 D.pre_ln ? mw.enc_lne_b : nullptr, P.enc_tok, 0, n, B.ra);
-  if (!grid_barrier(B.bar, tgt, status)) return;
   for (int l = 0; l < D.Le; ++l) {
     const EncLayerW<W>& L = mw.enc[l];
-    const W *g1, *b1;
-    float* st1;
-    const float* res1;
-    if (D.pre_ln) { g1 = L.ln1g; b1 = L.ln1b; st1 = nullptr; res1 = B.ra; }
-    else if (l == 0) { g1 = nullptr; b1 = nullptr; st1 = nullptr; res1 = B.ra; }
-    else { g1 = mw.enc[l - 1].ln2g; b1 = mw.enc[l - 1].ln2b; st1 = B.xa; res1 = B.xa; }
+    prefetch_gemm_weights(L.wqkv, 3 * D.d, D.d);
+    prefetch_gemm_weights(L.wo, D.d, D.d);
+    prefetch_gemm_weights(L.w1, D.f, D.d);
+    prefetch_gemm_weights(L.w2, D.d, D.f);
+  }
+  for (int l = 0; l < D.Ld; ++l) prefetch_gemm_weights(mw.dec[l].wkvc, 2 * D.d, D.d);
+
+  for (int l = 0; l < D.Le; ++l) {
+    const EncLayerW<W>& L = mw.enc[l];
     GemmArgs<W> g{};
-    g.M = n; g.N = 3 * D.d; g.K = D.d; g.x_src = B.ra; g.x_g = g1; g.x_b = b1; g.x_store = st1;
+    g.M = n; g.N = 3 * D.d; g.K = D.d;
+    if (l == 0) {
+      g.emb_tok = P.enc_tok; g.emb_pos0 = 0; g.x_store = B.ra;
+      if (pre) { g.ln_a_g = mw.enc_lne_g; g.ln_a_b = mw.enc_lne_b; g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
+    } else {
+      g.x_src = B.ra;
+      if (pre) { g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
+      else { g.ln_a_g = mw.enc[l - 1].ln2g; g.ln_a_b = mw.enc[l - 1].ln2b; g.x_store = B.xa; }
+    }
+    const float* res1 = (pre || l == 0) ? B.ra : B.xa;
     g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
     g.kdst_f = B.k; g.vdst_f = B.v;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
     attn_phase<float>(D, B.q, B.k, B.v, B.att, n, -1, n, scratch);
@@ -363,40 +410,39 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     g = GemmArgs<W>{};
     g.M = n; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
     g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
-    const W* g2 = D.pre_ln ? L.ln2g : L.ln1g;
-    const W* b2 = D.pre_ln ? L.ln2b : L.ln1b;
-    float* st2 = D.pre_ln ? nullptr : B.xb;
-    const float* res2 = D.pre_ln ? B.rb : B.xb;
     g = GemmArgs<W>{};
-    g.M = n; g.N = D.f; g.K = D.d; g.x_src = B.rb; g.x_g = g2; g.x_b = b2; g.x_store = st2;
+    g.M = n; g.N = D.f; g.K = D.d; g.x_src = B.rb;
+    if (pre) { g.ln_b_g = L.ln2g; g.ln_b_b = L.ln2b; }
+    else { g.ln_a_g = L.ln1g; g.ln_a_b = L.ln1b; g.x_store = B.xb; }
+    const float* res2 = pre ? B.rb : B.xb;
     g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
     g = GemmArgs<W>{};
     g.M = n; g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
     g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res2;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
   }
   // cross-attention keys and values of every decoder layer from the encoder output
   for (int l = 0; l < D.Ld; ++l) {
     GemmArgs<W> g{};
     g.M = n; g.N = 2 * D.d; g.K = D.d; g.x_src = B.ra;
-    g.x_g = D.pre_ln ? mw.enc_lnf_g : mw.enc[D.Le - 1].ln2g;
-    g.x_b = D.pre_ln ? mw.enc_lnf_b : mw.enc[D.Le - 1].ln2b;
+    g.ln_b_g = pre ? mw.enc_lnf_g : mw.enc[D.Le - 1].ln2g;
+    g.ln_b_b = pre ? mw.enc_lnf_b : mw.enc[D.Le - 1].ln2b;
     g.w = mw.dec[l].wkvc; g.bias = mw.dec[l].bkvc; g.epi = EPI_KVCROSS;
     g.kdst = B.kcross + (size_t)l * D.max_src * D.d;
     g.vdst = B.vcross + (size_t)l * D.max_src * D.d;
-    g.kv_ld = D.max_src;
-    gemm_phase<W>(g, D, smem);
+    gemm_phase<W>(g, T, D, smem);
   }
 }
 
 }  // namespace pd
+
 
 // ============================================================================================
 // host side
@@ -446,7 +492,8 @@ bool valid_config(const pd_config* c, std::string* why) {
   auto bad = [&](const char* m) { if (why) *why = m; return false; };
   if (!c) return bad("cfg is NULL");
   if (c->dtype != PD_DTYPE_F32 && c->dtype != PD_DTYPE_BF16) return bad("dtype");
-  if (c->d_model <= 0 || c->d_model % 256) return bad("d_model must be a positive multiple of 256");
+  if (c->d_model <= 0 || c->d_model % 256 || c->d_model > 1024)
+    return bad("d_model must be 256, 512, 768 or 1024");
   if (c->d_ff <= 0 || c->d_ff % 256) return bad("d_ff must be a positive multiple of 256");
   if (c->n_heads <= 0 || c->d_model % c->n_heads) return bad("n_heads must divide d_model");
   const int dh = c->d_model / c->n_heads;
@@ -530,6 +577,14 @@ pd_status dalloc(pd_ctx* c, T** p, size_t count) {
     if (s_ != PD_OK) return s_;    \
   } while (0)
 
+pd_status raise_smem_limit(pd_ctx* c, const void* fn) {
+  cudaFuncAttributes a{};
+  PD_CUDA(c, cudaFuncGetAttributes(&a, fn));
+  if ((size_t)a.maxDynamicSharedSizeBytes < c->smem)
+    PD_CUDA(c, cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->smem));
+  return PD_OK;
+}
+
 template <typename W>
 pd_status create_impl(pd_ctx* c, const void* weights) {
   const pd_config& cfg = c->cfg;
@@ -575,19 +630,25 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
   PD_TRY(dalloc(c, &B.trace, (size_t)D.max_tgt));
   PD_TRY(dalloc(c, &B.trace_tok, (size_t)D.max_tgt * D.max_tgt));
   PD_TRY(dalloc(c, &B.trace_prob, (size_t)D.max_tgt * D.max_tgt));
-  PD_TRY(dalloc(c, &B.bar, 2));
+  PD_TRY(dalloc(c, &B.bar, 4));
   PD_TRY(dalloc(c, &B.src, (size_t)D.max_src));
   PD_TRY(dalloc(c, &B.dbg_tok, (size_t)D.max_tgt));
+  PD_TRY(dalloc(c, &B.pos_tab, R * d));
+  if (!cfg.learned_pos) {
+    pd::sinusoid_kernel<<<c->n_sm, 256, 0, c->stream>>>(B.pos_tab, (int)R, (int)d);
+    PD_CUDA(c, cudaGetLastError());
+    PD_CUDA(c, cudaStreamSynchronize(c->stream));
+    c->launches += 1;
+  }
   PD_TRY(dalloc(c, &c->d_out_y, (size_t)D.max_tgt));
   PD_TRY(dalloc(c, &c->d_out_info, 4));
   PD_CUDA(c, cudaMemset(B.st, 0, sizeof(pd::DecState)));
-  PD_CUDA(c, cudaMemset(B.bar, 0, 2 * sizeof(unsigned)));
+  PD_CUDA(c, cudaMemset(B.bar, 0, 4 * sizeof(unsigned)));
 
   c->smem = pd::smem_layout(D, sizeof(W)).total;
-  PD_CUDA(c, cudaFuncSetAttribute(pd::decode_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)c->smem));
-  PD_CUDA(c, cudaFuncSetAttribute(pd::encode_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)c->smem));
+  // the limit is per kernel function and shared by every context of the process: only raise it
+  PD_TRY(raise_smem_limit(c, (const void*)pd::decode_kernel<W>));
+  PD_TRY(raise_smem_limit(c, (const void*)pd::encode_kernel<W>));
   int nb1 = 0, nb2 = 0;
   PD_CUDA(c, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb1, pd::decode_kernel<W>, pd::kThreads,
                                                            c->smem));
@@ -609,7 +670,7 @@ pd::KParams<W> base_params(pd_ctx* c) {
 
 template <typename W>
 pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P) {
-  PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).bar, 0, 2 * sizeof(unsigned), c->stream));
+  PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).bar, 0, 4 * sizeof(unsigned), c->stream));
   if (encode) PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).st, 0, sizeof(pd::DecState), c->stream));
   void* args[] = {&P};
   const void* fn = encode ? (const void*)pd::encode_kernel<W> : (const void*)pd::decode_kernel<W>;
@@ -847,6 +908,15 @@ pd_status pd_debug_logits(pd_ctx* c, const int32_t* y_in, int len, float* logits
 }
 
 void* pd_stream(pd_ctx* c) { return c ? (void*)c->stream : nullptr; }
+
+#ifdef PD_PHASE_TIMING
+// Development builds only: point the device phase timer at a buffer of 2 * cap uint64.
+int pd_debug_set_prof(void* dptr, int cap) {
+  if (cudaMemcpyToSymbol(pd::g_prof, &dptr, sizeof(dptr)) != cudaSuccess) return -3;
+  if (cudaMemcpyToSymbol(pd::g_prof_cap, &cap, sizeof(cap)) != cudaSuccess) return -3;
+  return 0;
+}
+#endif
 
 int64_t pd_launch_count(const pd_ctx* c) { return c ? c->launches : 0; }
 

@@ -20,9 +20,10 @@
 
 namespace pd {
 
-constexpr int kThreads = 512;
+constexpr int kThreads = 384;
 constexpr int kWarps = kThreads / 32;
-constexpr int kMTile = 16;          // rows per GEMM tile
+constexpr int kMTile = 8;           // rows per GEMM tile
+constexpr int kNCol = 4;            // output columns per warp iteration (kNCol * kMTile == 32)
 constexpr int kMaxLayers = 16;
 constexpr unsigned long long kWaitNs = 10000000000ull;  // bounded device waits: 10 s
 
@@ -97,6 +98,7 @@ struct Bufs {
   unsigned* bar;               // [0] barrier counter, [1] abort flag
   int* src;                    // [max_src]
   int* dbg_tok;                // [max_tgt]
+  float* pos_tab;              // sinusoidal positions [rows][d] (built once at create)
 };
 
 // ------------------------------------------------------------------------------------------
@@ -160,78 +162,123 @@ __device__ __forceinline__ float act_fn(float v, int act) {
 }
 
 // ------------------------------------------------------------------------------------------
-// grid barrier with a bounded wait
+// grid barriers with bounded waits
 // ------------------------------------------------------------------------------------------
 
-// All CTAs of the (cooperatively launched, hence co-resident) grid meet here.  The counter
-// only grows; `target` tracks how far it must have grown.  A CTA that waits longer than
-// kWaitNs raises the abort flag and records PD_ETIMEOUT; every CTA leaves on abort, so a
-// broken schedule ends the kernel instead of hanging the GPU.  Returns false on abort.
+#ifdef PD_PHASE_TIMING
+// Development-only phase timer: last arrival and release time of every barrier.
+__device__ unsigned long long* g_prof = nullptr;
+__device__ int g_prof_cap = 0;
+#define PD_PROF_ARRIVE(target)                                                             \
+  do {                                                                                     \
+    const int pidx_ = (int)((target) / gridDim.x);                                         \
+    if (g_prof != nullptr && pidx_ < g_prof_cap) atomicMax(&g_prof[2 * pidx_], globaltimer_ns()); \
+  } while (0)
+#define PD_PROF_RELEASE(target)                                                            \
+  do {                                                                                     \
+    const int pidx_ = (int)((target) / gridDim.x);                                         \
+    if (g_prof != nullptr && pidx_ < g_prof_cap && blockIdx.x == 0)                        \
+      g_prof[2 * pidx_ + 1] = globaltimer_ns();                                            \
+  } while (0)
+#else
+#define PD_PROF_ARRIVE(target) do { } while (0)
+#define PD_PROF_RELEASE(target) do { } while (0)
+#endif
+
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned atom_acq_rel_add(unsigned* p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v)
+               : "memory");
+  return old;
+}
+__device__ __forceinline__ void st_release_u32(unsigned* p, unsigned v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Bar words: [0] arrival counter (only grows), [1] abort flag, [2] release word of the
+// commit barrier.  Spin until *word >= target; give up after kWaitNs, raising the abort flag
+// and PD_ETIMEOUT, so that a broken schedule ends the kernel instead of hanging the GPU.
+__device__ __forceinline__ int spin_until(unsigned* bar, const unsigned* word, unsigned target,
+                                          int* status) {
+  const unsigned long long t0 = globaltimer_ns();
+  while (ld_acquire_u32(word) < target) {
+    if (ld_acquire_u32(bar + 1) != 0u) return 0;
+    if (globaltimer_ns() - t0 > kWaitNs) {
+      atomicExch(bar + 1, 1u);
+      atomicCAS(status, 0, (int)PD_ETIMEOUT);
+      return 0;
+    }
+  }
+  return 1;
+}
+
+// All CTAs of the (cooperatively launched, hence co-resident) grid meet here.  Release /
+// acquire at GPU scope: the bar.sync before the release-add orders every thread's writes of
+// this CTA before the arrival; the acquire load plus the bar.sync after it order the other
+// CTAs' writes before every thread's later reads.  Returns false on abort.
 __device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, int* status) {
   __shared__ int s_ok;
   __syncthreads();
   target += gridDim.x;
   if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(bar, 1u);
-    int ok = 1;
-    const unsigned long long t0 = globaltimer_ns();
-    while (ld_acquire_u32(bar) < target) {
-      if (ld_acquire_u32(bar + 1) != 0u) { ok = 0; break; }
-      if (globaltimer_ns() - t0 > kWaitNs) {
-        atomicExch(bar + 1, 1u);
-        atomicCAS(status, 0, (int)PD_ETIMEOUT);
-        ok = 0;
-        break;
-      }
-    }
-    __threadfence();
-    s_ok = ok;
+    PD_PROF_ARRIVE(target);
+    red_release_add(bar, 1u);
+    s_ok = spin_until(bar, bar, target, status);
+    PD_PROF_RELEASE(target);
   }
   __syncthreads();
   return s_ok != 0;
 }
 
-// ------------------------------------------------------------------------------------------
-// embedding: x = E[tok] * sqrt(d) + pos(p)  (+ embedding LayerNorm for pre-LN models)
-// ------------------------------------------------------------------------------------------
+// A barrier whose last arriving CTA runs `last()` before anybody is released: it sees every
+// CTA's writes (acq_rel arrival) and its own writes are released with the release word.
+// Folds the fixed-point commit into the LM-head barrier.  Returns false on abort.
+template <typename F>
+__device__ __forceinline__ bool grid_barrier_last(unsigned* bar, unsigned& target, int* status,
+                                                  F&& last) {
+  __shared__ int s_ok, s_last;
+  __syncthreads();
+  target += gridDim.x;
+  if (threadIdx.x == 0) {
+    PD_PROF_ARRIVE(target);
+    const unsigned old = atom_acq_rel_add(bar, 1u);
+    s_last = old + 1u == target;
+    s_ok = 1;
+  }
+  __syncthreads();
+  if (s_last) {
+    last();
+    __syncthreads();
+    if (threadIdx.x == 0) st_release_u32(bar + 2, target);
+  } else if (threadIdx.x == 0) {
+    s_ok = spin_until(bar, bar + 2, target, status);
+  }
+  if (threadIdx.x == 0) PD_PROF_RELEASE(target);
+  __syncthreads();
+  return s_ok != 0;
+}
 
-template <typename W>
-__device__ void embed_phase(const Dims& D, const W* __restrict__ E, const W* __restrict__ P,
-                            const W* lng, const W* lnb, const int* tok, int pos0, int M,
-                            float* out) {
-  const int lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * kWarps + (threadIdx.x >> 5);
-  const int tw = gridDim.x * kWarps;
-  for (int m = gw; m < M; m += tw) {
-    int t = __ldcg(tok + m);
-    t = t < 0 ? 0 : (t >= D.V ? D.V - 1 : t);
-    const int p = pos0 + m;
-    float* o = out + (size_t)m * D.d;
-    const int half = D.d / 2;
-    for (int e = lane; e < D.d; e += 32) {
-      float v = to_f(E[(size_t)t * D.d + e]) * D.emb_scale;
-      if (D.learned_pos) {
-        v += to_f(P[(size_t)(p < D.max_pos ? p : D.max_pos - 1) * D.d + e]);
-      } else {
-        const int kk = e < half ? e : e - half;
-        const double w = exp(-(2.0 * kk / D.d) * log(10000.0));
-        const double a = (double)p * w;
-        v += (float)(e < half ? sin(a) : cos(a));
-      }
-      o[e] = v;
-    }
-    if (lng != nullptr) {
-      __syncwarp();
-      float s = 0.f;
-      for (int e = lane; e < D.d; e += 32) s += o[e];
-      const float mean = warp_sum(s) / D.d;
-      float s2 = 0.f;
-      for (int e = lane; e < D.d; e += 32) { const float c = o[e] - mean; s2 += c * c; }
-      const float rstd = 1.0f / sqrtf(warp_sum(s2) / D.d + D.eps);
-      for (int e = lane; e < D.d; e += 32)
-        o[e] = (o[e] - mean) * rstd * to_f(lng[e]) + to_f(lnb[e]);
-    }
+// Ask L2 to fetch [p, p + bytes) ahead of use (no data returns to the SM).  The weights of a
+// phase do not depend on activations, so each CTA requests its own rows of the next phase
+// before it waits at the barrier, overlapping the HBM latency with the wait.
+__device__ __forceinline__ void l2_prefetch(const void* p, unsigned bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+// Sinusoidal position table, row p = [sin(p w_k) | cos(p w_k)], w_k = 10000^(-2k/d), in double
+// precision rounded to fp32 (run once when a context is created).
+__global__ void sinusoid_kernel(float* tab, int rows, int d) {
+  const int half = d / 2;
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < rows * d;
+       idx += gridDim.x * blockDim.x) {
+    const int p = idx / d, e = idx - p * d;
+    const int k = e < half ? e : e - half;
+    const double w = exp(-(2.0 * k / d) * log(10000.0));
+    const double a = (double)p * w;
+    tab[idx] = (float)(e < half ? sin(a) : cos(a));
   }
 }
 
@@ -242,9 +289,15 @@ __device__ void embed_phase(const Dims& D, const W* __restrict__ E, const W* __r
 template <typename W>
 struct GemmArgs {
   int M, N, K;
-  const float* x_src;       // [M][K] fp32 rows
-  const W *x_g, *x_b;       // LayerNorm of the input rows (nullptr: none)
-  float* x_store;           // write the normalised fp32 input rows here (nullptr: no)
+  // input rows X[M][K]: x_src rows, or (emb_tok != nullptr) the token embedding
+  // E[tok] * sqrt(d) + position(pos0 + m); then optionally LayerNorm ln_a, the result stored
+  // to x_store (fp32, by CTA 0), then optionally LayerNorm ln_b; X is rounded to W.
+  const float* x_src;
+  const int* emb_tok;
+  int emb_pos0;
+  const W *ln_a_g, *ln_a_b;
+  float* x_store;
+  const W *ln_b_g, *ln_b_b;
   const W* w;               // [N][K]
   const W* bias;            // [N] or nullptr
   int epi;
@@ -254,87 +307,237 @@ struct GemmArgs {
   W *kdst, *vdst;           // QKV: cache rows (slot = slot0 + m); KVCROSS: cross caches
   float *kdst_f, *vdst_f;   // QKV into fp32 buffers (encoder)
   int slot0;
-  int kv_ld;                // KVCROSS: rows per layer in the cross cache (max_src)
   Partial* part;            // ARGMAX: [grid][rows_ld]
   int part_ld;
 };
 
-// One output column for up to kMTile rows: each lane walks its K-chunks in ascending order,
-// then a fixed xor-butterfly; every lane ends with the same sums.
-__device__ __forceinline__ void dot_col(const __nv_bfloat16* __restrict__ wrow,
-                                        const __nv_bfloat16* xs, int K, int mt,
-                                        float (&acc)[kMTile]) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int r = 0; r < kMTile; ++r) acc[r] = 0.f;
-#pragma unroll 2
-  for (int k0 = lane * 8; k0 < K; k0 += 256) {
-    float w[8];
-    unpack8(ldg_nc_v4(wrow + k0), w);
-#pragma unroll
-    for (int r = 0; r < kMTile; ++r) {
-      if (r < mt) {
-        float x[8];
-        unpack8(*reinterpret_cast<const uint4*>(xs + (size_t)r * K + k0), x);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc[r] = fmaf(w[e], x[e], acc[r]);
-      }
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < kMTile; ++r) acc[r] = warp_sum(acc[r]);
-}
-
-__device__ __forceinline__ void dot_col(const float* __restrict__ wrow, const float* xs, int K,
-                                        int mt, float (&acc)[kMTile]) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int r = 0; r < kMTile; ++r) acc[r] = 0.f;
-#pragma unroll 2
-  for (int k0 = lane * 4; k0 < K; k0 += 128) {
-    const uint4 wu = ldg_nc_v4(wrow + k0);
-    const float w[4] = {__uint_as_float(wu.x), __uint_as_float(wu.y), __uint_as_float(wu.z),
-                        __uint_as_float(wu.w)};
-#pragma unroll
-    for (int r = 0; r < kMTile; ++r) {
-      if (r < mt) {
-        const float4 x = *reinterpret_cast<const float4*>(xs + (size_t)r * K + k0);
-        acc[r] = fmaf(w[0], x.x, acc[r]);
-        acc[r] = fmaf(w[1], x.y, acc[r]);
-        acc[r] = fmaf(w[2], x.z, acc[r]);
-        acc[r] = fmaf(w[3], x.w, acc[r]);
-      }
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < kMTile; ++r) acc[r] = warp_sum(acc[r]);
-}
-
-// Stage rows m0..m0+mt of the (optionally LayerNorm-ed) input into shared memory, rounded
-// to the weight type.  CTA 0 also writes the fp32 normalised rows to x_store.
+// Embedding and position tables (read by the GEMM whose input is the embedding).
 template <typename W>
-__device__ void stage_x(const GemmArgs<W>& g, float eps, int m0, int mt, W* xs) {
+struct EmbedTabs {
+  const W* E;               // token embedding [V][d]
+  const W* P;               // learned positions [max_pos][d] (or nullptr)
+  const float* ptab;        // sinusoidal positions [rows][d] (or nullptr)
+};
+
+// Reduce-scatter of 32 per-lane partial sums: afterwards lane L holds the warp total of value
+// L.  Every value is summed over the lanes by the same balanced tree (pairs at lane distance
+// 16, 8, 4, 2, 1), so the result of a value does not depend on its index.
+__device__ __forceinline__ float reduce_scatter32(float (&v)[32]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int s = 16; s >= 1; s >>= 1) {
+    const bool upper = (lane & s) != 0;
+#pragma unroll
+    for (int j = 0; j < s; ++j) {
+      const float send = upper ? v[j] : v[j + s];
+      const float keep = upper ? v[j + s] : v[j];
+      v[j] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+    }
+  }
+  return v[0];
+}
+
+// Elements one warp covers per 16-byte load of every lane (one "K-step").
+template <typename W> struct KStep { static constexpr int E = 32 * 16 / (int)sizeof(W); };
+
+// Partial dot products of kNCol output columns n0.. for up to kMTile rows over the K-steps
+// s0..s0+ns-1 (ns <= 2): all weight loads of the warp are issued before the first FMA, each
+// element is accumulated in ascending K order, then the reduce-scatter leaves value
+// (column c, row r) on lane c * kMTile + r.
+__device__ __forceinline__ float dot_part(const __nv_bfloat16* __restrict__ w, int K, int n0,
+                                          int nvalid, const __nv_bfloat16* xs, int mt, int s0,
+                                          int ns) {
+  const int lane = threadIdx.x & 31;
+  uint4 wr[2][kNCol];
+#pragma unroll
+  for (int t = 0; t < 2; ++t)
+#pragma unroll
+    for (int c = 0; c < kNCol; ++c)
+      wr[t][c] = (t < ns && c < nvalid)
+                     ? ldg_nc_v4(w + (size_t)(n0 + c) * K + (s0 + t) * 256 + lane * 8)
+                     : make_uint4(0u, 0u, 0u, 0u);
+  float acc[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+#pragma unroll
+  for (int t = 0; t < 2; ++t) {
+    if (t < ns) {
+      float wv[kNCol][8];
+#pragma unroll
+      for (int c = 0; c < kNCol; ++c) unpack8(wr[t][c], wv[c]);
+#pragma unroll
+      for (int r = 0; r < kMTile; ++r) {
+        if (r < mt) {
+          float x[8];
+          unpack8(*reinterpret_cast<const uint4*>(xs + (size_t)r * K + (s0 + t) * 256 + lane * 8), x);
+#pragma unroll
+          for (int c = 0; c < kNCol; ++c)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[c * kMTile + r] = fmaf(wv[c][e], x[e], acc[c * kMTile + r]);
+        }
+      }
+    }
+  }
+  return reduce_scatter32(acc);
+}
+
+__device__ __forceinline__ float dot_part(const float* __restrict__ w, int K, int n0, int nvalid,
+                                          const float* xs, int mt, int s0, int ns) {
+  const int lane = threadIdx.x & 31;
+  uint4 wr[2][kNCol];
+#pragma unroll
+  for (int t = 0; t < 2; ++t)
+#pragma unroll
+    for (int c = 0; c < kNCol; ++c)
+      wr[t][c] = (t < ns && c < nvalid)
+                     ? ldg_nc_v4(w + (size_t)(n0 + c) * K + (s0 + t) * 128 + lane * 4)
+                     : make_uint4(0u, 0u, 0u, 0u);
+  float acc[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+#pragma unroll
+  for (int t = 0; t < 2; ++t) {
+    if (t < ns) {
+#pragma unroll
+      for (int r = 0; r < kMTile; ++r) {
+        if (r < mt) {
+          const float4 x =
+              *reinterpret_cast<const float4*>(xs + (size_t)r * K + (s0 + t) * 128 + lane * 4);
+#pragma unroll
+          for (int c = 0; c < kNCol; ++c) {
+            float& a = acc[c * kMTile + r];
+            a = fmaf(__uint_as_float(wr[t][c].x), x.x, a);
+            a = fmaf(__uint_as_float(wr[t][c].y), x.y, a);
+            a = fmaf(__uint_as_float(wr[t][c].z), x.z, a);
+            a = fmaf(__uint_as_float(wr[t][c].w), x.w, a);
+          }
+        }
+      }
+    }
+  }
+  return reduce_scatter32(acc);
+}
+
+constexpr int kMaxRowRegs = 8;      // embedded / normalised rows: <= 8 float4 per lane
+
+// LayerNorm of a row held as float4 v[i] = elements lane*4 + 128*i: mean and biased variance
+// from per-lane sums in ascending i, then fixed butterflies.
+template <typename W>
+__device__ __forceinline__ void ln_regs(float4 (&v)[kMaxRowRegs], int nI, int K, const W* g,
+                                        const W* b, float eps) {
+  const int lane = threadIdx.x & 31;
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < kMaxRowRegs; ++i)
+    if (i < nI) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+  const float mean = warp_sum(s) / K;
+  float s2 = 0.f;
+#pragma unroll
+  for (int i = 0; i < kMaxRowRegs; ++i) {
+    if (i < nI) {
+      const float a = v[i].x - mean, bb = v[i].y - mean, c = v[i].z - mean, d = v[i].w - mean;
+      s2 += (a * a + bb * bb) + (c * c + d * d);
+    }
+  }
+  const float rstd = 1.0f / sqrtf(warp_sum(s2) / K + eps);
+#pragma unroll
+  for (int i = 0; i < kMaxRowRegs; ++i) {
+    if (i < nI) {
+      const int k = lane * 4 + 128 * i;
+      v[i].x = (v[i].x - mean) * rstd * to_f(g[k]) + to_f(b[k]);
+      v[i].y = (v[i].y - mean) * rstd * to_f(g[k + 1]) + to_f(b[k + 1]);
+      v[i].z = (v[i].z - mean) * rstd * to_f(g[k + 2]) + to_f(b[k + 2]);
+      v[i].w = (v[i].w - mean) * rstd * to_f(g[k + 3]) + to_f(b[k + 3]);
+    }
+  }
+}
+
+__device__ __forceinline__ void put4(float* xs, float4 v) { *reinterpret_cast<float4*>(xs) = v; }
+__device__ __forceinline__ void put4(__nv_bfloat16* xs, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *reinterpret_cast<unsigned*>(&a);
+  u.y = *reinterpret_cast<unsigned*>(&b);
+  *reinterpret_cast<uint2*>(xs) = u;
+}
+
+template <typename W>
+__device__ __forceinline__ float4 get4(const W* p) {
+  return make_float4(to_f(p[0]), to_f(p[1]), to_f(p[2]), to_f(p[3]));
+}
+
+// Stage rows m0..m0+mt of the GEMM input into shared memory (one warp per row, each element
+// loaded once into registers).
+template <typename W>
+__device__ void stage_x(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims& D, int m0,
+                        int mt, W* xs) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int K = g.K;
+  const bool any_ln = g.ln_a_g != nullptr || g.ln_b_g != nullptr || g.emb_tok != nullptr;
   for (int r = warp; r < mt; r += kWarps) {
-    const float* src = g.x_src + (size_t)(m0 + r) * K;
-    float mean = 0.f, rstd = 1.f;
-    if (g.x_g != nullptr) {
-      float s = 0.f;
-      for (int e = lane; e < K; e += 32) s += __ldcg(src + e);
-      mean = warp_sum(s) / K;
-      float s2 = 0.f;
-      for (int e = lane; e < K; e += 32) { const float c = __ldcg(src + e) - mean; s2 += c * c; }
-      rstd = 1.0f / sqrtf(warp_sum(s2) / K + eps);
-    }
+    const int m = m0 + r;
     const bool store = g.x_store != nullptr && blockIdx.x == 0;
-    for (int e = lane; e < K; e += 32) {
-      float v = __ldcg(src + e);
-      if (g.x_g != nullptr) v = (v - mean) * rstd * to_f(g.x_g[e]) + to_f(g.x_b[e]);
-      if (store) g.x_store[(size_t)(m0 + r) * K + e] = v;
-      xs[(size_t)r * K + e] = from_f<W>(v);
+    if (!any_ln) {                       // plain copy (any K multiple of 128)
+      const float* src = g.x_src + (size_t)m * K;
+      for (int k = lane * 4; k < K; k += 128) {
+        const float4 v = *reinterpret_cast<const float4*>(src + k);
+        if (store) *reinterpret_cast<float4*>(g.x_store + (size_t)m * K + k) = v;
+        put4(xs + (size_t)r * K + k, v);
+      }
+      continue;
     }
+    const int nI = K / 128;              // K <= 1024 for rows that are embedded or normalised
+    float4 v[kMaxRowRegs];
+    if (g.emb_tok != nullptr) {
+      int t = g.emb_tok[m];
+      t = t < 0 ? 0 : (t >= D.V ? D.V - 1 : t);
+      const int p = g.emb_pos0 + m;
+      const W* er = T.E + (size_t)t * K;
+#pragma unroll
+      for (int i = 0; i < kMaxRowRegs; ++i) {
+        if (i < nI) {
+          const int k = lane * 4 + 128 * i;
+          const float4 e = get4(er + k);
+          float4 ps;
+          if (T.P != nullptr) ps = get4(T.P + (size_t)(p < D.max_pos ? p : D.max_pos - 1) * K + k);
+          else ps = *reinterpret_cast<const float4*>(T.ptab + (size_t)p * K + k);
+          v[i] = make_float4(e.x * D.emb_scale + ps.x, e.y * D.emb_scale + ps.y,
+                             e.z * D.emb_scale + ps.z, e.w * D.emb_scale + ps.w);
+        }
+      }
+    } else {
+      const float* src = g.x_src + (size_t)m * K;
+#pragma unroll
+      for (int i = 0; i < kMaxRowRegs; ++i)
+        if (i < nI) v[i] = *reinterpret_cast<const float4*>(src + lane * 4 + 128 * i);
+    }
+    if (g.ln_a_g != nullptr) ln_regs(v, nI, K, g.ln_a_g, g.ln_a_b, D.eps);
+    if (store) {
+#pragma unroll
+      for (int i = 0; i < kMaxRowRegs; ++i)
+        if (i < nI)
+          *reinterpret_cast<float4*>(g.x_store + (size_t)m * K + lane * 4 + 128 * i) = v[i];
+    }
+    if (g.ln_b_g != nullptr) ln_regs(v, nI, K, g.ln_b_g, g.ln_b_b, D.eps);
+#pragma unroll
+    for (int i = 0; i < kMaxRowRegs; ++i)
+      if (i < nI) put4(xs + (size_t)r * K + lane * 4 + 128 * i, v[i]);
+  }
+}
+
+// Bulk L2 prefetch of the weight rows this CTA's warps will read in a GEMM phase over N
+// columns of K (the same column groups gemm_phase assigns them).
+template <typename W>
+__device__ __forceinline__ void prefetch_gemm_weights(const W* w, int N, int K) {
+  if (w == nullptr) return;
+  const int ngroups = (N + kNCol - 1) / kNCol;
+  for (int gi = blockIdx.x + (int)(threadIdx.x >> 5) * gridDim.x; gi < ngroups;
+       gi += gridDim.x * kWarps) {
+    if ((threadIdx.x & 31) != 0) continue;
+    const int n0 = gi * kNCol;
+    const int nv = N - n0 < kNCol ? N - n0 : kNCol;
+    l2_prefetch(w + (size_t)n0 * K, (unsigned)(nv * K * sizeof(W)));
   }
 }
 
@@ -366,72 +569,90 @@ __device__ __forceinline__ void partial_merge(Partial& a, const Partial& b) {
   }
 }
 
+// GEMM phase.  N is cut into column groups of kNCol; a group is computed by kw warps of one
+// CTA, warp j covering K-steps 2j and 2j+1 (kw = ceil(K-steps / 2), a function of K only),
+// and their partial sums are added in warp order.  Groups are dealt to CTAs round robin
+// (group g -> CTA g mod grid), so that even a 512-column phase spreads over 128 SMs.
 template <typename W>
-__device__ void gemm_phase(const GemmArgs<W>& g, const Dims& D, unsigned char* smem) {
+__device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>& T,
+                                        const Dims& D, unsigned char* smem) {
   W* xs = reinterpret_cast<W*>(smem);
-  Partial* ps = reinterpret_cast<Partial*>(smem + (size_t)kMTile * (D.d > D.f ? D.d : D.f) *
-                                                      sizeof(W));
+  unsigned char* small = smem + (size_t)kMTile * (D.d > D.f ? D.d : D.f) * sizeof(W);
+  Partial* ps = reinterpret_cast<Partial*>(small);        // [kWarps][32]
+  float* red = reinterpret_cast<float*>(small);           // [kWarps][32] (not used with ps)
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  const int gw = blockIdx.x * kWarps + warp;
-  const int tw = gridDim.x * kWarps;
+  const int steps = g.K / KStep<W>::E;
+  const int kw = (steps + 1) / 2;
+  const int gpc = kWarps / kw;
+  const int slot = warp / kw, part = warp - slot * kw;
+  const int s0 = 2 * part, ns = steps - s0 < 2 ? steps - s0 : 2;
+  const int ngroups = (g.N + kNCol - 1) / kNCol;
+  const int stride = gridDim.x * gpc;
+  const int c = lane / kMTile, r = lane % kMTile;   // the (column, row) this lane finishes
   for (int m0 = 0; m0 < g.M; m0 += kMTile) {
     const int mt = g.M - m0 < kMTile ? g.M - m0 : kMTile;
     __syncthreads();
-    stage_x(g, D.eps, m0, mt, xs);
+    stage_x(g, T, D, m0, mt, xs);
     __syncthreads();
     float amx = -INFINITY, asum = 0.f;
     int aidx = 0x7fffffff, anan = 0;
-    for (int n = gw; n < g.N; n += tw) {
-      float acc[kMTile];
-      dot_col(g.w + (size_t)n * g.K, xs, g.K, mt, acc);
-      // lane r finishes row r (a compile-time-indexed select keeps acc in registers)
+    for (int base = 0; base < ngroups; base += stride) {
+      const int gi = base + slot * gridDim.x + blockIdx.x;
+      const bool active = slot < gpc && gi < ngroups;
+      const int n0 = gi * kNCol;
+      const int nvalid = active ? (g.N - n0 < kNCol ? g.N - n0 : kNCol) : 0;
       float a = 0.f;
-#pragma unroll
-      for (int r = 0; r < kMTile; ++r)
-        if (lane == r) a = acc[r];
-      if (lane < mt) {
-      const int m = m0 + lane;
+      if (active) a = dot_part(g.w, g.K, n0, nvalid, xs, mt, s0, ns);
+      if (kw > 1) {
+        if (active) red[warp * 32 + lane] = a;
+        __syncthreads();
+        if (active && part == 0)
+          for (int j = 1; j < kw; ++j) a += red[(warp + j) * 32 + lane];
+        __syncthreads();
+      }
+      if (!active || part != 0 || r >= mt || c >= nvalid) continue;
+      const int m = m0 + r, n = n0 + c;
       const float bias = g.bias != nullptr ? to_f(g.bias[n]) : 0.f;
       const float v = a + bias;
       switch (g.epi) {
         case EPI_STORE: g.out[(size_t)m * g.ld + n] = v; break;
         case EPI_ACT: g.out[(size_t)m * g.ld + n] = act_fn(v, D.act); break;
-        case EPI_RESID:
-          g.out[(size_t)m * g.ld + n] = v + __ldcg(g.resid + (size_t)m * g.ld + n);
-          break;
+        case EPI_RESID: g.out[(size_t)m * g.ld + n] = v + g.resid[(size_t)m * g.ld + n]; break;
         case EPI_QKV: {
-          const int which = n / D.d, c = n - which * D.d;
+          const int which = n / D.d, cc = n - which * D.d;
           if (which == 0) {
-            g.out[(size_t)m * D.d + c] = v;
+            g.out[(size_t)m * D.d + cc] = v;
           } else if (g.kdst != nullptr) {
             W* dst = which == 1 ? g.kdst : g.vdst;
-            dst[(size_t)(g.slot0 + m) * D.d + c] = from_f<W>(v);
+            dst[(size_t)(g.slot0 + m) * D.d + cc] = from_f<W>(v);
           } else {
             float* dst = which == 1 ? g.kdst_f : g.vdst_f;
-            dst[(size_t)m * D.d + c] = v;
+            dst[(size_t)m * D.d + cc] = v;
           }
           break;
         }
         case EPI_KVCROSS: {
-          const int layer = n / (2 * D.d), c2 = n - layer * 2 * D.d;
-          const int which = c2 / D.d, c = c2 - which * D.d;
-          W* dst = (which == 0 ? g.kdst : g.vdst) + (size_t)layer * g.kv_ld * D.d;
-          dst[(size_t)m * D.d + c] = from_f<W>(v);
+          const int which = n / D.d, cc = n - which * D.d;
+          W* dst = which == 0 ? g.kdst : g.vdst;
+          dst[(size_t)m * D.d + cc] = from_f<W>(v);
           break;
         }
         case EPI_ARGMAX: argmax_push(v, n, amx, aidx, asum, anan); break;
         case EPI_LOGITS: g.out[(size_t)m * g.ld + n] = v; break;
       }
-      }
     }
     if (g.epi == EPI_ARGMAX) {
-      // combine the warps of this CTA in warp order, then publish the CTA partial per row
-      if (lane < kMTile) ps[warp * kMTile + lane] = Partial{amx, aidx, asum, anan};
+      // lane c*kMTile + r of a part-0 warp holds row r over its columns n0 + c: merge in warp
+      // order, then lane (column) order, and publish the CTA partial per row
+      __syncthreads();
+      ps[warp * 32 + lane] = Partial{amx, aidx, asum, anan};
       __syncthreads();
       if (warp == 0 && lane < mt) {
         Partial acc = ps[lane];
-        for (int w2 = 1; w2 < kWarps; ++w2) partial_merge(acc, ps[w2 * kMTile + lane]);
+        for (int w2 = 0; w2 < kWarps; ++w2)
+          for (int c2 = 0; c2 < kNCol; ++c2)
+            if (w2 != 0 || c2 != 0) partial_merge(acc, ps[w2 * 32 + c2 * kMTile + lane]);
         g.part[(size_t)blockIdx.x * g.part_ld + m0 + lane] = acc;
       }
     }
@@ -451,7 +672,7 @@ __device__ __forceinline__ float key_dot<__nv_bfloat16>(const __nv_bfloat16* kro
   float s = 0.f;
   for (int e = 0; e < dh; e += 8) {
     float k[8];
-    unpack8(__ldcg(reinterpret_cast<const uint4*>(krow + e)), k);
+    unpack8(*reinterpret_cast<const uint4*>(krow + e), k);
 #pragma unroll
     for (int t = 0; t < 8; ++t) s = fmaf(qs[e + t], k[t], s);
   }
@@ -462,7 +683,7 @@ template <>
 __device__ __forceinline__ float key_dot<float>(const float* krow, const float* qs, int dh) {
   float s = 0.f;
   for (int e = 0; e < dh; e += 4) {
-    const float4 k = __ldcg(reinterpret_cast<const float4*>(krow + e));
+    const float4 k = *reinterpret_cast<const float4*>(krow + e);
     s = fmaf(qs[e], k.x, s);
     s = fmaf(qs[e + 1], k.y, s);
     s = fmaf(qs[e + 2], k.z, s);
@@ -471,19 +692,37 @@ __device__ __forceinline__ float key_dot<float>(const float* krow, const float* 
   return s;
 }
 
-__device__ __forceinline__ float ld_kv(const float* p) { return __ldcg(p); }
-__device__ __forceinline__ float ld_kv(const __nv_bfloat16* p) {
-  const unsigned short u = __ldcg(reinterpret_cast<const unsigned short*>(p));
-  return __uint_as_float(((unsigned)u) << 16);
+// acc[e] += p * v[e] for 32 consecutive value elements of one key.
+__device__ __forceinline__ void add_pv32(const __nv_bfloat16* v, float p, float (&acc)[32]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float f[8];
+    unpack8(*reinterpret_cast<const uint4*>(v + 8 * i), f);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[8 * i + e] = fmaf(p, f[e], acc[8 * i + e]);
+  }
+}
+__device__ __forceinline__ void add_pv32(const float* v, float p, float (&acc)[32]) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 f = *reinterpret_cast<const float4*>(v + 4 * i);
+    acc[4 * i] = fmaf(p, f.x, acc[4 * i]);
+    acc[4 * i + 1] = fmaf(p, f.y, acc[4 * i + 1]);
+    acc[4 * i + 2] = fmaf(p, f.z, acc[4 * i + 2]);
+    acc[4 * i + 3] = fmaf(p, f.w, acc[4 * i + 3]);
+  }
 }
 
+// One warp per (row m, head): lane l owns keys l, l+32, ...  Scores, softmax and the
+// p-weighted value sums are accumulated per lane in ascending key order, then combined by
+// fixed butterflies, so a row's result depends only on its own query and keys.
 // causal_pos0 >= 0: row m attends keys 0..causal_pos0+m; else all n_keys keys.
 template <typename KV>
-__device__ void attn_phase(const Dims& D, const float* q, const KV* kc, const KV* vc,
+__device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV* kc, const KV* vc,
                            float* out, int M, int causal_pos0, int n_keys, float* scratch) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  const int gw = blockIdx.x * kWarps + warp;
+  const int gw = warp * gridDim.x + blockIdx.x;     // items dealt to CTAs round robin
   const int tw = gridDim.x * kWarps;
   const int dh = D.dh;
   float* qs = scratch + (size_t)warp * (128 + D.rows + 4);
@@ -492,7 +731,7 @@ __device__ void attn_phase(const Dims& D, const float* q, const KV* kc, const KV
   for (int it = gw; it < M * D.H; it += tw) {
     const int m = it / D.H, h = it - m * D.H;
     const int T = causal_pos0 >= 0 ? causal_pos0 + m + 1 : n_keys;
-    for (int e = lane; e < dh; e += 32) qs[e] = __ldcg(q + (size_t)m * D.d + h * dh + e) * scale;
+    for (int e = lane; e < dh; e += 32) qs[e] = q[(size_t)m * D.d + h * dh + e] * scale;
     __syncwarp();
     float lmax = -INFINITY;
     for (int j = lane; j < T; j += 32) {
@@ -508,12 +747,16 @@ __device__ void attn_phase(const Dims& D, const float* q, const KV* kc, const KV
       lsum += p;
     }
     const float sum = warp_sum(lsum);
-    __syncwarp();
-    for (int e = lane; e < dh; e += 32) {
-      float acc = 0.f;
-      const KV* vp = vc + h * dh + e;
-      for (int j = 0; j < T; ++j) acc = fmaf(ps[j], ld_kv(vp + (size_t)j * D.d), acc);
-      out[(size_t)m * D.d + h * dh + e] = acc / sum;
+    for (int c0 = 0; c0 < dh; c0 += 32) {
+      float acc[32];
+#pragma unroll
+      for (int e = 0; e < 32; ++e) acc[e] = 0.f;
+      for (int j = lane; j < T; j += 32) {
+        const float p = ps[j];
+        add_pv32(vc + (size_t)j * D.d + h * dh + c0, p, acc);
+      }
+      const float tot = reduce_scatter32(acc);
+      out[(size_t)m * D.d + h * dh + c0 + lane] = tot / sum;
     }
     __syncwarp();
   }

@@ -351,3 +351,17 @@ def test_nan_weights_give_enan():
         with pytest.raises(pkg.PdError) as e:
             d.decode("greedy", 4)
         assert e.value.status == -5                                 # PD_ENAN
+
+
+def test_two_contexts_interleaved(tiny, marian):
+    """Contexts with different sizes stay usable side by side (per-function launch limits
+    are process-wide)."""
+    small = pkg.Decoder(pkg.Config.from_spec(synth.TINY, 8, 8), tiny.w.blob)
+    src = synth.TINY_JACOBI.sentences()[0]
+    small.encode(src[:8])
+    tiny.dec.encode(src)
+    a = tiny.dec.decode("jacobi", 16)
+    b = small.decode("jacobi", 8)
+    assert tiny.dec.decode("greedy", 16).tokens == a.tokens
+    assert small.decode("greedy", 8).tokens == b.tokens
+    small.close()
