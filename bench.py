@@ -192,7 +192,7 @@ def run_gpu(args):
 
     spec = WORKLOAD.spec
     weights = synth.make_weights(spec, seed=WORKLOAD.weight_seed)
-    sents = WORKLOAD.sentences()
+    sents = WORKLOAD.sentences()[:args.sentences] if args.sentences else WORKLOAD.sentences()
     n_s = len(sents)
     max_src = max(len(s) for s in sents)
     max_tgt = max(WORKLOAD.max_len(len(s)) for s in sents)
@@ -313,7 +313,8 @@ def run_gpu(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic: seeded N(0,0.02) weights, uniform random source ids",
-            "config": {"workload": WORKLOAD.name, "sentences_per_step": n_s,
+            "config": {"workload": WORKLOAD.name if n_s == WORKLOAD.n_sentences else
+                       f"{WORKLOAD.name} (first {n_s} sentences only)", "sentences_per_step": n_s,
                        "timing": "CUDA events on the library stream; L2 flushed (256 MB write) "
                                  "between steps; replicas across GPUs"},
             "greedy": {"value": greedy_tps, "unit": "tokens/s",
@@ -345,6 +346,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sentences", type=int, default=0,
+                    help="use only the first N sentences of the workload (profiling runs)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
