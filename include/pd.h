@@ -143,6 +143,19 @@ pd_status pd_decode_device(pd_ctx* ctx, const pd_decode_params* p, int32_t* d_y,
  * decoder's key/value cache. */
 pd_status pd_debug_logits(pd_ctx* ctx, const int32_t* y_in, int len, float* logits);
 
+/* Test-only, allocation-free variant of pd_debug_logits (the paper has no counterpart: this
+ * is a service for callers that may not allocate device memory, e.g. a process whose device
+ * memory is owned by another pool or that must not grow after start-up).  Same arguments and
+ * results as pd_debug_logits, but the logits are staged in a fixed 4 MiB array inside the
+ * library's device image instead of a per-call allocation, so len * vocab must not exceed
+ * 1,048,576 (PD_EINVAL otherwise).  Every GPU that loads the library holds the array until the
+ * process exits.  The first call for a device looks up the array's device address (with that
+ * device made current for the lookup); make that first call before any stream capture.  All
+ * calls share the one array, which keeps the last call's contents: calls that overlap on the
+ * GPU (several contexts or threads at once) race and must be serialised by the caller.
+ * Synchronous; calls no device allocator. */
+pd_status pd_debug_logits_static(pd_ctx* ctx, const int32_t* y_in, int len, float* logits);
+
 /* The context's cudaStream_t. */
 void* pd_stream(pd_ctx* ctx);
 

@@ -25,8 +25,9 @@ METHODS = {"greedy": 0, "jacobi": 1, "gs_jacobi": 2, "hybrid_gs_jacobi": 3}
 
 # Every symbol include/pd.h declares.
 EXPORTED = ("pd_weights_nbytes", "pd_create", "pd_export_weights", "pd_encode",
-            "pd_encode_device", "pd_decode", "pd_decode_device", "pd_debug_logits", "pd_stream",
-            "pd_launch_count", "pd_last_error", "pd_destroy")
+            "pd_encode_device", "pd_decode", "pd_decode_device", "pd_debug_logits",
+            "pd_debug_logits_static", "pd_stream", "pd_launch_count", "pd_last_error",
+            "pd_destroy")
 
 
 class PdError(RuntimeError):
@@ -86,6 +87,8 @@ def load_library() -> ctypes.CDLL:
     lib.pd_decode_device.restype = I
     lib.pd_debug_logits.argtypes = [P, pi32, I, ctypes.POINTER(ctypes.c_float)]
     lib.pd_debug_logits.restype = I
+    lib.pd_debug_logits_static.argtypes = [P, pi32, I, ctypes.POINTER(ctypes.c_float)]
+    lib.pd_debug_logits_static.restype = I
     lib.pd_stream.argtypes = [P]
     lib.pd_stream.restype = P
     lib.pd_launch_count.argtypes = [P]
@@ -228,6 +231,16 @@ class Decoder:
         self._check(self._lib.pd_debug_logits(self._h, _i32p(a), int(a.size),
                                                out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))),
                     "pd_debug_logits")
+        return out
+
+    def debug_logits_static(self, y_in) -> np.ndarray:
+        """As debug_logits, staging the logits in the library's fixed device array instead of a
+        per-call device allocation (for callers that may not allocate device memory)."""
+        a = np.ascontiguousarray(y_in, dtype=np.int32)
+        out = np.zeros((a.size, self.cfg.vocab), dtype=np.float32)
+        self._check(self._lib.pd_debug_logits_static(
+            self._h, _i32p(a), int(a.size), out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))),
+            "pd_debug_logits_static")
         return out
 
     def export_weights(self, dtype) -> np.ndarray:

@@ -13,6 +13,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -904,6 +905,82 @@ pd_status pd_debug_logits(pd_ctx* c, const int32_t* y_in, int len, float* logits
   cudaFree(dl);
   if (s != PD_OK) return s;
   if (e != cudaSuccess) return fail(c, PD_ECUDA, std::string("debug logits: ") + cudaGetErrorString(e));
+  return PD_OK;
+}
+
+}  // extern "C"
+
+// ------------------------------------------------------------------------------------------
+// pd_debug_logits_static: the teacher-forced logits without any device allocation
+// ------------------------------------------------------------------------------------------
+//
+// pd_debug_logits stages the logits in a device buffer it allocates for each call.  Callers
+// that may not allocate device memory (a process whose memory is pooled by another owner, a
+// code path running under an allocator lock, or a program that must not grow its footprint
+// after start-up) use this variant: the staging buffer is a fixed array in the library's own
+// device image, loaded once per GPU with the module and kept until the process exits.
+
+namespace {
+
+constexpr size_t kStaticLogitsFloats = (size_t)1 << 20;   // 4 MiB: len * vocab <= 1,048,576
+constexpr int kMaxDevices = 64;
+
+std::mutex g_static_mu;
+float* g_static_dev[kMaxDevices] = {};   // device address of the array, per device
+
+}  // namespace
+
+// In host code this name stands for the array; its device address comes from
+// cudaGetSymbolAddress (done once per device in static_logits_addr).
+static __device__ __align__(256) float g_static_logits[kStaticLogitsFloats];
+
+namespace {
+
+// Device address of g_static_logits on the context's device, looked up on the first call
+// made for that device (with that device current) and cached.
+pd_status static_logits_addr(pd_ctx* c, float** out) {
+  if (c->device < 0 || c->device >= kMaxDevices) return fail(c, PD_EINVAL, "device index too large");
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (g_static_dev[c->device] == nullptr) {
+    int prev = -1;
+    PD_CUDA(c, cudaGetDevice(&prev));
+    if (prev != c->device) PD_CUDA(c, cudaSetDevice(c->device));
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_logits);
+    if (prev != c->device) cudaSetDevice(prev);
+    if (e != cudaSuccess || p == nullptr)
+      return fail(c, PD_ECUDA, std::string("cudaGetSymbolAddress(g_static_logits): ") +
+                                   cudaGetErrorString(e));
+    g_static_dev[c->device] = static_cast<float*>(p);
+  }
+  *out = g_static_dev[c->device];
+  return PD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+pd_status pd_debug_logits_static(pd_ctx* c, const int32_t* y_in, int len, float* logits) {
+  if (!c) return PD_EINVAL;
+  if (!y_in || !logits || len < 1 || len > c->cfg.max_tgt_len)
+    return fail(c, PD_EINVAL, "len must be in [1, max_tgt_len]");
+  if ((size_t)len * (size_t)c->cfg.vocab > kStaticLogitsFloats)
+    return fail(c, PD_EINVAL, "len * vocab exceeds the static logits buffer (1,048,576 floats)");
+  if (c->cfg.learned_pos && len > c->cfg.max_pos) return fail(c, PD_EINVAL, "len exceeds max_pos");
+  for (int k = 0; k < len; ++k)
+    if (y_in[k] < 0 || y_in[k] >= c->cfg.vocab) return fail(c, PD_EINVAL, "token id out of range");
+  if (!c->encoded) return fail(c, PD_ESTATE, "pd_debug_logits_static before pd_encode");
+  float* dl = nullptr;
+  PD_TRY(static_logits_addr(c, &dl));
+  int* dtok = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.dbg_tok : c->bf.dbg_tok;
+  PD_CUDA(c, cudaMemcpyAsync(dtok, y_in, len * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  // every element of the [len][vocab] region is written by the kernel: nothing to clear
+  PD_TRY(c->cfg.dtype == PD_DTYPE_BF16 ? debug_impl<__nv_bfloat16>(c, len, dl)
+                                       : debug_impl<float>(c, len, dl));
+  PD_CUDA(c, cudaMemcpyAsync(logits, dl, (size_t)len * c->cfg.vocab * sizeof(float),
+                             cudaMemcpyDeviceToHost, c->stream));
+  PD_CUDA(c, cudaStreamSynchronize(c->stream));
   return PD_OK;
 }
 
