@@ -31,6 +31,23 @@ WORKLOAD = synth.MARIAN_GS
 METRIC = "translated tokens/s at batch 1, GS-Jacobi vs greedy AR; HBM GB/s % of peak"
 FALLBACK_HBM_GBS = 6800.0
 
+# DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
+# ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel sources whose
+# SHA-256 is recorded here; any other source reports traffic null.
+DRAM_BYTES_PER_PASS = 33.8e6
+DRAM_SOURCES_SHA256 = "3e050957c3e621e3e5ec32b16cefd6894404053548a0e38ae7dd17863bff22ea"
+
+
+def kernel_sources_sha256() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2305_10427_gb300", "csrc")
+    for f in sorted(os.listdir(d)):
+        if f.endswith((".cu", ".cuh")):
+            h.update(f.encode())
+            h.update(open(os.path.join(d, f), "rb").read())
+    return h.hexdigest()
+
 
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -278,6 +295,9 @@ def run_gpu(args):
     dec_s_per_step = dec_ms / args.steps / 1e3
     achieved = total_bytes / dec_s_per_step / 1e9
     peak, peak_kind = peaks()
+    traffic = None                                  # per average decode launch
+    if DRAM_SOURCES_SHA256 and kernel_sources_sha256() == DRAM_SOURCES_SHA256:
+        traffic = DRAM_BYTES_PER_PASS * passes / n_s
 
     # end to end through the host API
     e2e_tok, h2d, d2h = 0, 0, 0
@@ -322,7 +342,8 @@ def run_gpu(args):
             "passes_per_token": passes / max(1, sum(toks)),
             "us_per_pass": 1e6 * dec_s_per_step / max(1, passes),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None,
+                         "frac": achieved / peak, "traffic": traffic,
+                         "algorithmic_bytes_per_launch": total_bytes / n_s,
                          "kernel": "decode_kernel<bf16>", "peak_kind": peak_kind},
             "e2e": {"value": e2e_tps, "unit": "tokens/s", "h2d_bytes_per_step": h2d // args.steps,
                     "d2h_bytes_per_step": d2h // args.steps},
