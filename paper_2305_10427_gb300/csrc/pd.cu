@@ -11,6 +11,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstddef>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -47,7 +48,7 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   L.part = L.xs + ((size_t)kMTile * kmax * wsize + 15) / 16 * 16;
   L.scratch = L.part + (size_t)kWarps * 32 * sizeof(Partial);
   L.commit = L.scratch + (size_t)kWarps * (128 + D.rows + 4) * sizeof(float);
-  L.total = L.commit + (size_t)(D.max_tgt + 1) * 2 * sizeof(int) + 64;
+  L.total = L.commit + (size_t)(D.max_tgt + 1) * 3 * sizeof(int) + 64;
   return L;
 }
 
@@ -192,6 +193,9 @@ __device__ __forceinline__ Partial shfl_partial(const Partial& a, int o) {
   return b;
 }
 
+// The decoding state is copied into shared memory with one load per field (issued together),
+// the block's previous draft likewise; one thread then takes the decisions from shared memory
+// and the results are written back in parallel.
 template <typename W>
 __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   const Dims& D = P.D;
@@ -199,12 +203,17 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   const SmemLayout SL = smem_layout(D, sizeof(W));
   int* ntok = reinterpret_cast<int*>(smem + SL.commit);
   float* nprob = reinterpret_cast<float*>(ntok + D.max_tgt + 1);
-  __shared__ int s_nan;
-  volatile DecState* s = B.st;
-  const int blk = s->blk;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) s_nan = 0;
+  int* yold = reinterpret_cast<int*>(nprob + D.max_tgt + 1);
+  constexpr int kNS = (int)(sizeof(DecState) / sizeof(int));
+  __shared__ DecState ss;
+  __shared__ int s_nan, s_eos;
+  const int tid = threadIdx.x;
+  const int lane = tid & 31, warp = tid >> 5;
+  if (tid < kNS) reinterpret_cast<int*>(&ss)[tid] = __ldcg(reinterpret_cast<const int*>(B.st) + tid);
+  if (tid == 0) { s_nan = 0; s_eos = 0x7fffffff; }
   __syncthreads();
+  const int blk = ss.blk, i = ss.i;
+  for (int r = tid; r < blk; r += blockDim.x) yold[r] = __ldcg(B.y + i + r);
   // per row: the CTA partials merged lane-wise in ascending CTA order, then by a fixed
   // butterfly (the merge is symmetric, so every lane ends with the same result)
   for (int r = warp; r < blk; r += kWarps) {
@@ -222,73 +231,88 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
     }
   }
   __syncthreads();
-  if (threadIdx.x != 0) return;
-
-  int* y = B.y;
-  const int i = s->i;
-  int c = 0;
-  while (c < blk && ntok[c] == y[i + c]) ++c;
-  const int stop = c == blk;
-  int eos_idx = -1;
-  for (int r = 0; r < blk; ++r)
-    if (ntok[r] == D.eos) { eos_idx = r; break; }
-  for (int r = 0; r < blk; ++r) y[i + r] = ntok[r];
-  s->k = s->k + 1;
-  const int n_it = s->n_iters + 1;
-  s->n_iters = n_it;
-  const int t = s->n_trace;
-  if (t < D.max_tgt) {
-    pd_trace_step row;
-    row.step = n_it; row.block_start = i; row.block_len = blk; row.n_converged = c;
-    row.stop = stop; row.eos_idx = eos_idx;
-    B.trace[t] = row;
-    for (int r = 0; r < blk; ++r) {
+  const int t = ss.n_trace;
+  for (int r = tid; r < blk; r += blockDim.x) {
+    B.y[i + r] = ntok[r];
+    if (t < D.max_tgt) {
       B.trace_tok[(size_t)t * D.max_tgt + r] = ntok[r];
       B.trace_prob[(size_t)t * D.max_tgt + r] = nprob[r];
     }
-    s->n_trace = t + 1;
   }
-  if (s_nan) { s->status = PD_ENAN; s->n_y = i - 1; s->done = 1; return; }
-
-  if (stop || s->k >= blk) {                       // the block is solved
-    const bool one_pos = s->method == PD_GREEDY || s->ar_tail;
-    if (one_pos) {
-      const bool eos_ends = s->ar_tail ? true : (s->stop_at_eos != 0);
-      if (eos_ends && ntok[0] == D.eos) { s->n_y = i; s->done = 1; }
-    } else if (s->method == PD_HYBRID_GS_JACOBI && eos_idx >= 0) {
-      s->n_y = i + eos_idx;                        // through the EOS (Algorithm 3)
-      s->done = 1;
+  bool scan = false;                                // search y_1..y_m for the first EOS
+  if (tid == 0) {
+    int c = 0;
+    while (c < blk && ntok[c] == yold[c]) ++c;
+    const int stop = c == blk;
+    int eos_idx = -1;
+    for (int r = 0; r < blk; ++r)
+      if (ntok[r] == D.eos) { eos_idx = r; break; }
+    ss.k = ss.k + 1;
+    const int n_it = ss.n_iters + 1;
+    ss.n_iters = n_it;
+    if (t < D.max_tgt) {
+      pd_trace_step row;
+      row.step = n_it; row.block_start = i; row.block_len = blk; row.n_converged = c;
+      row.stop = stop; row.eos_idx = eos_idx;
+      B.trace[t] = row;
+      ss.n_trace = t + 1;
     }
-    if (!s->done) {
-      const int ni = i + blk;
-      if (s->method == PD_HYBRID_GS_JACOBI && !s->ar_tail && ni > s->h) {
-        s->ar_tail = 1;                            // greedy tail up to max_len
-        s->b_eff = 1;
-        s->m_eff = s->max_len;
-      }
-      if (ni > s->m_eff) {
-        s->done = 1;
-        int n = s->m_eff;
-        if ((s->method == PD_JACOBI || s->method == PD_GS_JACOBI) && s->stop_at_eos) {
-          for (int p = 1; p <= s->m_eff; ++p)
-            if (y[p] == D.eos) { n = p; break; }
+    if (s_nan) {
+      ss.status = PD_ENAN; ss.n_y = i - 1; ss.done = 1;
+    } else {
+      if (stop || ss.k >= blk) {                   // the block is solved
+        const bool one_pos = ss.method == PD_GREEDY || ss.ar_tail;
+        if (one_pos) {
+          const bool eos_ends = ss.ar_tail ? true : (ss.stop_at_eos != 0);
+          if (eos_ends && ntok[0] == D.eos) { ss.n_y = i; ss.done = 1; }
+        } else if (ss.method == PD_HYBRID_GS_JACOBI && eos_idx >= 0) {
+          ss.n_y = i + eos_idx;                    // through the EOS (Algorithm 3)
+          ss.done = 1;
         }
-        s->n_y = n;
-      } else {
-        s->i = ni;
-        const int rest = s->m_eff - ni + 1;
-        s->blk = s->b_eff < rest ? s->b_eff : rest;
-        s->k = 0;
+        if (!ss.done) {
+          const int ni = i + blk;
+          if (ss.method == PD_HYBRID_GS_JACOBI && !ss.ar_tail && ni > ss.h) {
+            ss.ar_tail = 1;                        // greedy tail up to max_len
+            ss.b_eff = 1;
+            ss.m_eff = ss.max_len;
+          }
+          if (ni > ss.m_eff) {
+            ss.done = 1;
+            ss.n_y = ss.m_eff;
+            scan = (ss.method == PD_JACOBI || ss.method == PD_GS_JACOBI) && ss.stop_at_eos;
+          } else {
+            ss.i = ni;
+            const int rest = ss.m_eff - ni + 1;
+            ss.blk = ss.b_eff < rest ? ss.b_eff : rest;
+            ss.k = 0;
+          }
+        }
+      }
+      // the pass budget, and a hard cap no correct schedule reaches (at most m passes for the
+      // parallel part plus max_len for a greedy tail): the loop can never run away
+      if (!ss.done && ((ss.max_passes > 0 && n_it >= ss.max_passes) || n_it > 2 * ss.max_len + 2)) {
+        ss.status = PD_ENOTCONV;
+        ss.n_y = ss.i - 1;
+        ss.done = 1;
       }
     }
+    if (scan) s_eos = -1;                          // ask for the scan below
   }
-  // the pass budget, and a hard cap no correct schedule reaches (at most m passes for the
-  // parallel part plus max_len for a greedy tail): the loop can never run away
-  if (!s->done && ((s->max_passes > 0 && n_it >= s->max_passes) || n_it > 2 * s->max_len + 2)) {
-    s->status = PD_ENOTCONV;
-    s->n_y = s->i - 1;
-    s->done = 1;
+  __syncthreads();
+  if (s_eos == -1) {                               // first EOS among y_1..y_m (written above)
+    __syncthreads();
+    if (tid == 0) s_eos = 0x7fffffff;
+    __syncthreads();
+    for (int p = 1 + tid; p <= ss.m_eff; p += blockDim.x)
+      if (__ldcg(B.y + p) == D.eos) atomicMin(&s_eos, p);
+    __syncthreads();
+    if (tid == 0 && s_eos != 0x7fffffff) ss.n_y = s_eos;
+    __syncthreads();
   }
+  // write the state back; a non-zero status is only ever set, never cleared
+  if (tid < kNS && tid != (int)(offsetof(DecState, status) / sizeof(int)))
+    reinterpret_cast<int*>(B.st)[tid] = reinterpret_cast<const int*>(&ss)[tid];
+  if (tid == 0 && ss.status != 0) atomicCAS(&B.st->status, 0, ss.status);
 }
 
 template <typename W>

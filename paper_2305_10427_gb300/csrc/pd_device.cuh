@@ -582,12 +582,15 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
   float* red = reinterpret_cast<float*>(small);           // [kWarps][32] (not used with ps)
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
+  // K-steps per warp: 1 when the phase then still fits in one round over the grid (shorter
+  // dot chains for the small GEMMs), else 2.  A function of N, K and the grid only.
   const int steps = g.K / KStep<W>::E;
-  const int kw = (steps + 1) / 2;
+  const int ngroups = (g.N + kNCol - 1) / kNCol;
+  const int spw = (steps <= kWarps && ngroups <= (int)gridDim.x * (kWarps / steps)) ? 1 : 2;
+  const int kw = (steps + spw - 1) / spw;
   const int gpc = kWarps / kw;
   const int slot = warp / kw, part = warp - slot * kw;
-  const int s0 = 2 * part, ns = steps - s0 < 2 ? steps - s0 : 2;
-  const int ngroups = (g.N + kNCol - 1) / kNCol;
+  const int s0 = spw * part, ns = steps - s0 < spw ? steps - s0 : spw;
   const int stride = gridDim.x * gpc;
   const int c = lane / kMTile, r = lane % kMTile;   // the (column, row) this lane finishes
   for (int m0 = 0; m0 < g.M; m0 += kMTile) {
