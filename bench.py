@@ -34,8 +34,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
 # ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel sources whose
 # SHA-256 is recorded here; any other source reports traffic null.
-DRAM_BYTES_PER_PASS = 33.8e6
-DRAM_SOURCES_SHA256 = "3e050957c3e621e3e5ec32b16cefd6894404053548a0e38ae7dd17863bff22ea"
+DRAM_BYTES_PER_PASS = 29.9e6
+DRAM_SOURCES_SHA256 = "857e8c5220d4ea0b167edfa0f80eedc3ad47a89e093c3e11693301a45fa630e8"
 
 
 def kernel_sources_sha256() -> str:
@@ -77,6 +77,21 @@ def decode_bytes(spec, n_src, trace):
         i, blk = row["block_start"], row["block_len"]
         tot += pass_bytes(spec, i - 1 + blk, n_src, blk)
     return tot
+
+
+def over_ranks(x: float, op: str, dist=None, device="cpu") -> float:
+    """max or sum of a per-rank number over all ranks (identity without a process group)."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return x
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def job_rate(units: float, seconds: float, dist=None, device="cpu") -> float:
+    """Whole-job throughput of replicas: units done by all ranks / the slowest rank's time."""
+    return over_ranks(units, "sum", dist, device) / over_ranks(seconds, "max", dist, device)
 
 
 class Clocks:
@@ -158,7 +173,7 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    weights = synth.make_weights(WORKLOAD.spec, seed=WORKLOAD.weight_seed)
+    weights = WORKLOAD.weights()
     sents = WORKLOAD.sentences()
     # each step: GS-Jacobi (b=5) of the next sentence of the workload by the float64 oracle
     order = sorted(range(len(sents)), key=lambda k: len(sents[k]))[:args.warmup + args.steps]
@@ -208,7 +223,7 @@ def run_gpu(args):
         build.build(force=False)
 
     spec = WORKLOAD.spec
-    weights = synth.make_weights(spec, seed=WORKLOAD.weight_seed)
+    weights = WORKLOAD.weights()
     sents = WORKLOAD.sentences()[:args.sentences] if args.sentences else WORKLOAD.sentences()
     n_s = len(sents)
     max_src = max(len(s) for s in sents)
@@ -222,8 +237,10 @@ def run_gpu(args):
     d_y = torch.zeros((n_s, max_tgt), dtype=torch.int32, device="cuda")
     d_info = torch.zeros((n_s, 4), dtype=torch.int32, device="cuda")
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
-    params = {m: [pkg.Decoder.params(m, WORKLOAD.max_len(len(s)), b=WORKLOAD.b)
-                  for s in sents] for m in ("gs_jacobi", "greedy")}
+    params = {m: [pkg.Decoder.params(m, WORKLOAD.max_len(len(s)), b=b)
+                  for s in sents]
+              for m, b in (("gs_jacobi", WORKLOAD.b), ("greedy", 1), ("jacobi", 1),
+                           ("hybrid_gs_jacobi", 3))}
 
     def device_step(method, ev=None):
         for k in range(n_s):
@@ -259,18 +276,10 @@ def run_gpu(args):
         return tokens, total_ms, dec_ms, dec.launch_count - launches0, d_info.cpu().numpy()
 
     def max_over_ranks(x):
-        if dist is None:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return over_ranks(x, "max", dist, "cuda")
 
     def sum_over_ranks(x):
-        if dist is None:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t)
-        return float(t.item())
+        return over_ranks(x, "sum", dist, "cuda")
 
     # greedy AR reference point (same kernels, one position per pass)
     g_tok, g_ms, g_dec_ms, _, g_info = timed("greedy", args.steps, args.warmup)
@@ -281,6 +290,15 @@ def run_gpu(args):
         tok, ms, dec_ms, launches, info = timed("gs_jacobi", args.steps, args.warmup)
     ms_max = max_over_ranks(ms)
     tps = sum_over_ranks(tok) / (ms_max / 1e3)
+
+    # the other methods (one timed step each), for the report
+    others = {}
+    if args.all_methods:
+        for m in ("jacobi", "hybrid_gs_jacobi"):
+            t_tok, t_ms, _, _, t_info = timed(m, 1, 1)
+            others[m] = {"value": sum_over_ranks(t_tok) / (max_over_ranks(t_ms) / 1e3),
+                         "unit": "tokens/s",
+                         "passes_per_token": float(t_info[:, 1].sum()) / max(1, int(t_info[:, 0].sum()))}
 
     # roofline of the decode kernel: algorithmic bytes from the traces of one step
     total_bytes, passes = 0, 0
@@ -296,7 +314,8 @@ def run_gpu(args):
     achieved = total_bytes / dec_s_per_step / 1e9
     peak, peak_kind = peaks()
     traffic = None                                  # per average decode launch
-    if DRAM_SOURCES_SHA256 and kernel_sources_sha256() == DRAM_SOURCES_SHA256:
+    if (DRAM_SOURCES_SHA256 and kernel_sources_sha256() == DRAM_SOURCES_SHA256
+            and WORKLOAD is synth.MARIAN_GS):
         traffic = DRAM_BYTES_PER_PASS * passes / n_s
 
     # end to end through the host API
@@ -338,7 +357,8 @@ def run_gpu(args):
                        "timing": "CUDA events on the library stream; L2 flushed (256 MB write) "
                                  "between steps; replicas across GPUs"},
             "greedy": {"value": greedy_tps, "unit": "tokens/s",
-                       "gs_jacobi_speedup": tps / greedy_tps},
+                       "gs_jacobi_speedup": tps / greedy_tps,
+                       "passes_per_token": float(g_info[:, 1].sum()) / max(1, int(g_info[:, 0].sum()))},
             "passes_per_token": passes / max(1, sum(toks)),
             "us_per_pass": 1e6 * dec_s_per_step / max(1, passes),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
@@ -350,6 +370,8 @@ def run_gpu(args):
             "gpu_launches": launches,
             "clocks": clk.summary(),
         }
+        if others:
+            line["other_methods"] = others
         if cpu is not None:
             line["cpu_baseline"] = cpu
         print(json.dumps(line), flush=True)
@@ -367,9 +389,17 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="marian", choices=["marian", "marian-knob"],
+                    help="marian: the benchmark workload; marian-knob: the same model with a "
+                         "small token-embedding scale (Jacobi accepts several tokens per pass)")
+    ap.add_argument("--all-methods", action="store_true",
+                    help="also time full-sentence Jacobi and Hybrid GS-Jacobi (b=3), one step each")
     ap.add_argument("--sentences", type=int, default=0,
                     help="use only the first N sentences of the workload (profiling runs)")
     args = ap.parse_args()
+    global WORKLOAD
+    if args.workload == "marian-knob":
+        WORKLOAD = synth.MARIAN_KNOB
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

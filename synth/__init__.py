@@ -220,6 +220,10 @@ class Workload:
     b: int
     max_len_factor: int      # max_len = factor * src_len (0: max_len = fixed_max_len)
     fixed_max_len: int = 0
+    embed_std: float = None  # token-embedding scale of the weights (None: the weight std)
+
+    def weights(self) -> "Weights":
+        return make_weights(self.spec, seed=self.weight_seed, embed_std=self.embed_std)
 
     def sentences(self) -> List[np.ndarray]:
         return sentences(self.sentence_seed, self.n_sentences, self.len_lo, self.len_hi,
@@ -240,6 +244,12 @@ MARIAN_HYBRID = dataclasses.replace(MARIAN_GS, name="marian-base-bf16 hybrid_gs_
                                     method="hybrid_gs_jacobi", b=3)
 MARIAN_JACOBI = dataclasses.replace(MARIAN_GS, name="marian-base-bf16 jacobi b=max_len",
                                     method="jacobi", b=0)
+# The Marian-sized model with a 20x smaller token-embedding scale ("dependency knob"): its
+# predictions depend less on the previous token, so Jacobi iterations accept several positions
+# per pass -- the mechanism behind the paper's speedups, which random weights otherwise lack.
+MARIAN_KNOB = dataclasses.replace(
+    MARIAN_GS, name="marian-base-bf16 embed_std=0.001 gs_jacobi b=5, 256 sentences of 8..64 ids, "
+                    "max_len=2n", embed_std=0.001)
 # mBART-like bf16 model, 128 sentences of 16..128 ids, GS-Jacobi b=5 (and 16).
 MBART_GS = Workload("mbart-large-bf16 gs_jacobi b=5, 128 sentences of 16..128 ids, max_len=2n",
                     MBART, 0, 1, 128, 16, 128, "gs_jacobi", 5, 2)

@@ -365,3 +365,55 @@ def test_two_contexts_interleaved(tiny, marian):
     assert tiny.dec.decode("greedy", 16).tokens == a.tokens
     assert small.decode("greedy", 8).tokens == b.tokens
     small.close()
+
+
+# ---- pre-LN, GELU, learned positions (the mBART-style structure) at a small size -----------
+
+PRE_F32 = synth.small_spec("pre-gelu-learned-f32", d_model=256, n_heads=4, d_ff=512,
+                           n_enc_layers=2, n_dec_layers=2, vocab=3000,
+                           activation=synth.ACT_GELU, pre_ln=True, learned_pos=True, max_pos=128,
+                           dtype=synth.DTYPE_F32)
+PRE_BF16 = synth.small_spec("pre-gelu-learned-bf16", d_model=512, n_heads=8, d_ff=1024,
+                            n_enc_layers=2, n_dec_layers=3, vocab=5000,
+                            activation=synth.ACT_GELU, pre_ln=True, learned_pos=True, max_pos=128,
+                            dtype=synth.DTYPE_BF16)
+
+
+@pytest.fixture(scope="module")
+def pre_f32():
+    s = Setup(PRE_F32, 64, 64, seed=11, ln_noise=0.2, embed_std=0.05)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
+def pre_bf16():
+    s = Setup(PRE_BF16, 64, 64, seed=12, ln_noise=0.2, embed_std=0.05)
+    yield s
+    s.dec.close()
+
+
+@pytest.mark.parametrize("name", ["pre_f32", "pre_bf16"])
+def test_pre_ln_models(name, request):
+    """Pre-LN blocks with embedding and final LayerNorms, exact GELU and a learned position
+    table: logits against the oracle, every method bit-identical to the GPU's greedy, pass
+    counts and traces equal to the oracle's where its decisions had margin."""
+    s = request.getfixturevalue(name)
+    tol = 2e-2 if s.spec.dtype == synth.DTYPE_BF16 else 1e-4
+    rng = np.random.default_rng(21)
+    compared = 0
+    for src in synth.sentences(22, 3, 6, 24, s.spec.vocab):
+        s.dec.encode(src)
+        y_in = np.r_[synth.BOS_ID, rng.integers(0, s.spec.vocab, size=len(src))].astype(np.int32)
+        got = s.dec.debug_logits(y_in)
+        assert rel_row_err(got, s.model.logits(s.mem(src), y_in)).max() < tol
+        max_len = 2 * len(src)
+        res = all_methods(s.dec, max_len)
+        g = res["greedy"].tokens
+        for k, r in res.items():
+            assert r.tokens == g, k
+            assert r.n_iters <= max_len, k
+        check_tokens_teacher_forced(s, src, g)
+        compared += compare_with_oracle_runs(s, src, max_len, res)
+    if s.spec.dtype == synth.DTYPE_F32:
+        assert compared >= 3
