@@ -56,128 +56,178 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
 // one decoder pass over M rows (input tokens tok[0..M) at positions pos0..pos0+M-1)
 // ------------------------------------------------------------------------------------------
 
+// The weight-pointer table, copied into shared memory when a kernel starts: the acquire at
+// every grid barrier drops the SM's L1 copies of global data, so a table read from global
+// memory would cost an L2 round trip in every phase.
+template <typename W>
+__device__ __forceinline__ ModelW<W>& smem_mw() {
+  __shared__ ModelW<W> s;
+  return s;
+}
+template <typename W>
+__device__ __forceinline__ void load_smem_mw(const KParams<W>& P) {
+  static_assert(sizeof(ModelW<W>) % 8 == 0, "pointer table");
+  const unsigned long long* src = reinterpret_cast<const unsigned long long*>(P.mw);
+  unsigned long long* dst = reinterpret_cast<unsigned long long*>(&smem_mw<W>());
+  for (int i = threadIdx.x; i < (int)(sizeof(ModelW<W>) / 8); i += blockDim.x) dst[i] = src[i];
+  __syncthreads();
+}
+
 template <typename W>
 __device__ __forceinline__ EmbedTabs<W> embed_tabs(const KParams<W>& P) {
-  const ModelW<W>& mw = *P.mw;
+  const ModelW<W>& mw = smem_mw<W>();
   return EmbedTabs<W>{mw.embed, P.D.learned_pos ? mw.pos : nullptr,
                       P.D.learned_pos ? nullptr : P.B.pos_tab};
 }
 
-// Every weight row this CTA will read in one decoder pass, requested from L2 in phase order
-// at the start of the pass: HBM streams the pass's weights while the (latency-bound) chain
-// of phases runs, and each phase then finds its rows in L2.
+// Phases of a decoder pass, per layer in this order (the attention phases take scalar
+// arguments); phase 8 * Ld is the LM head.
+enum : int {
+  PH_QKV = 0, PH_SELF = 1, PH_O = 2, PH_QC = 3, PH_CROSS = 4, PH_OC = 5, PH_FFN1 = 6, PH_FFN2 = 7
+};
+
+__device__ __forceinline__ bool is_attn_phase(int ph, int nph) {
+  return ph < nph - 1 && ((ph & 7) == PH_SELF || (ph & 7) == PH_CROSS);
+}
+
+// Arguments of GEMM phase ph of a pass over M rows at positions pos0.. with input tokens tok;
+// the LM head (ph = 8 Ld) writes raw logits if logits != nullptr, else argmax partials.
 template <typename W>
-__device__ void prefetch_pass(const KParams<W>& P) {
+__device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const int* tok,
+                          float* logits, GemmArgs<W>& g) {
   const Dims& D = P.D;
-  const ModelW<W>& mw = *P.mw;
-  for (int l = 0; l < D.Ld; ++l) {
-    const DecLayerW<W>& L = mw.dec[l];
-    prefetch_gemm_weights(L.wqkv, 3 * D.d, D.d);
-    prefetch_gemm_weights(L.wo, D.d, D.d);
-    prefetch_gemm_weights(L.wqc, D.d, D.d);
-    prefetch_gemm_weights(L.woc, D.d, D.d);
-    prefetch_gemm_weights(L.w1, D.f, D.d);
-    prefetch_gemm_weights(L.w2, D.d, D.f);
+  const Bufs<W>& B = P.B;
+  const ModelW<W>& mw = smem_mw<W>();
+  const bool pre = D.pre_ln != 0;
+  g = GemmArgs<W>{};
+  g.M = M;
+  if (ph == 8 * D.Ld) {                 // LM head over the final hidden rows
+    g.N = D.V; g.K = D.d; g.x_src = B.ra;
+    g.ln_b_g = pre ? mw.dec_lnf_g : mw.dec[D.Ld - 1].ln3g;
+    g.ln_b_b = pre ? mw.dec_lnf_b : mw.dec[D.Ld - 1].ln3b;
+    g.w = mw.embed;
+    if (logits != nullptr) { g.epi = EPI_LOGITS; g.out = logits; g.ld = D.V; }
+    else { g.epi = EPI_ARGMAX; g.part = B.part; g.part_ld = D.rows; }
+    return;
   }
-  prefetch_gemm_weights(mw.embed, D.V, D.d);
+  const int l = ph >> 3;
+  const DecLayerW<W>& L = mw.dec[l];
+  switch (ph & 7) {
+    case PH_QKV:
+      // self-attention sublayer input.  Pre-LN: x = LN1(r), residual r.  Post-LN: x = the
+      // previous sublayer's LN of its output, which is also the residual; layer 0 takes the
+      // embedding as is.  The embedding is computed in this GEMM's prologue.
+      g.N = 3 * D.d; g.K = D.d;
+      if (l == 0) {
+        g.emb_tok = tok; g.emb_pos0 = pos0; g.x_store = B.ra;
+        if (pre) {
+          g.ln_a_g = mw.dec_lne_g; g.ln_a_b = mw.dec_lne_b; g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b;
+        }
+      } else {
+        g.x_src = B.ra;
+        if (pre) { g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
+        else { g.ln_a_g = mw.dec[l - 1].ln3g; g.ln_a_b = mw.dec[l - 1].ln3b; g.x_store = B.xa; }
+      }
+      g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
+      g.kdst = B.kself + (size_t)l * D.max_tgt * D.d;
+      g.vdst = B.vself + (size_t)l * D.max_tgt * D.d;
+      g.slot0 = pos0;
+      break;
+    case PH_O:                          // self-attention output + residual
+      g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
+      g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = (pre || l == 0) ? B.ra : B.xa;
+      break;
+    case PH_QC:                         // cross-attention query
+      g.N = D.d; g.K = D.d; g.x_src = B.rb;
+      if (pre) { g.ln_b_g = L.ln2g; g.ln_b_b = L.ln2b; }
+      else { g.ln_a_g = L.ln1g; g.ln_a_b = L.ln1b; g.x_store = B.xb; }
+      g.w = L.wqc; g.bias = L.bqc; g.epi = EPI_STORE; g.out = B.q; g.ld = D.d;
+      break;
+    case PH_OC:                         // cross-attention output + residual
+      g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.woc; g.bias = L.boc;
+      g.epi = EPI_RESID; g.out = B.rc; g.ld = D.d; g.resid = pre ? B.rb : B.xb;
+      break;
+    case PH_FFN1:
+      g.N = D.f; g.K = D.d; g.x_src = B.rc;
+      if (pre) { g.ln_b_g = L.ln3g; g.ln_b_b = L.ln3b; }
+      else { g.ln_a_g = L.ln2g; g.ln_a_b = L.ln2b; g.x_store = B.xc; }
+      g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
+      break;
+    case PH_FFN2:
+      g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
+      g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = pre ? B.rc : B.xc;
+      break;
+  }
+}
+
+// Ask L2 for the weight rows this CTA reads in GEMM phase ph (nothing for attention phases),
+// so that HBM streams them while the latency-bound chain of earlier phases runs.
+template <typename W>
+__device__ void prefetch_phase(const KParams<W>& P, int ph) {
+  const Dims& D = P.D;
+  const int nph = 8 * D.Ld + 1;
+  if (ph >= nph || is_attn_phase(ph, nph)) return;
+  const ModelW<W>& mw = smem_mw<W>();
+  if (ph == nph - 1) { prefetch_gemm_weights(mw.embed, D.V, D.d); return; }
+  const DecLayerW<W>& L = mw.dec[ph >> 3];
+  switch (ph & 7) {
+    case PH_QKV: prefetch_gemm_weights(L.wqkv, 3 * D.d, D.d); break;
+    case PH_O: prefetch_gemm_weights(L.wo, D.d, D.d); break;
+    case PH_QC: prefetch_gemm_weights(L.wqc, D.d, D.d); break;
+    case PH_OC: prefetch_gemm_weights(L.woc, D.d, D.d); break;
+    case PH_FFN1: prefetch_gemm_weights(L.w1, D.f, D.d); break;
+    case PH_FFN2: prefetch_gemm_weights(L.w2, D.d, D.f); break;
+  }
 }
 
 template <typename W>
-__device__ bool decoder_pass(const KParams<W>& P, int M, int pos0, const int* tok,
-                             unsigned& tgt, unsigned char* smem) {
+__device__ __forceinline__ GemmArgs<W>& smem_args() {
+  __shared__ GemmArgs<W> s;
+  return s;
+}
+
+// One decoder pass over M rows followed by the LM head, as a loop over phases separated by
+// grid barriers.  The arguments of the next GEMM phase are written to shared memory by one
+// thread while its CTA waits at the barrier, and the weights two phases ahead are requested
+// from L2 there, so that neither is on the chain of dependent phases.
+template <typename W>
+__device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, float* logits,
+                         unsigned& tgt, unsigned char* smem) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
-  const ModelW<W>& mw = *P.mw;
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
   const EmbedTabs<W> T = embed_tabs(P);
-  const bool pre = D.pre_ln != 0;
-
-  for (int l = 0; l < D.Ld; ++l) {
-    const DecLayerW<W>& L = mw.dec[l];
-    W* kc = B.kself + (size_t)l * D.max_tgt * D.d;
-    W* vc = B.vself + (size_t)l * D.max_tgt * D.d;
-    W* kx = B.kcross + (size_t)l * D.max_src * D.d;
-    W* vx = B.vcross + (size_t)l * D.max_src * D.d;
-
-    // self-attention sublayer input.  Pre-LN: x = LN1(r), residual r.  Post-LN: x = the
-    // previous sublayer's LN of its output, which is also the residual; layer 0 takes the
-    // embedding as is.  The embedding is computed in this GEMM's prologue.
-    GemmArgs<W> g{};
-    g.M = M; g.N = 3 * D.d; g.K = D.d;
-    if (l == 0) {
-      g.emb_tok = tok; g.emb_pos0 = pos0; g.x_store = B.ra;
-      if (pre) { g.ln_a_g = mw.dec_lne_g; g.ln_a_b = mw.dec_lne_b; g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
+  GemmArgs<W>& ga = smem_args<W>();
+  const int nph = 8 * D.Ld + 1;
+  if (threadIdx.x == 32) gemm_args(P, 0, M, pos0, tok, logits, ga);
+  prefetch_phase(P, 0);
+  prefetch_phase(P, 2);
+  prefetch_phase(P, nph - 1);
+  __syncthreads();
+  for (int ph = 0; ph < nph; ++ph) {
+    const bool attn = is_attn_phase(ph, nph);
+    if (attn) {
+      const int l = ph >> 3;
+      if ((ph & 7) == PH_SELF)
+        attn_phase<W>(D, B.q, B.kself + (size_t)l * D.max_tgt * D.d,
+                      B.vself + (size_t)l * D.max_tgt * D.d, B.att, M, pos0, 0, scratch);
+      else
+        attn_phase<W>(D, B.q, B.kcross + (size_t)l * D.max_src * D.d,
+                      B.vcross + (size_t)l * D.max_src * D.d, B.att, M, -1, P.n_src, scratch);
     } else {
-      g.x_src = B.ra;
-      if (pre) { g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
-      else { g.ln_a_g = mw.dec[l - 1].ln3g; g.ln_a_b = mw.dec[l - 1].ln3b; g.x_store = B.xa; }
+      gemm_phase<W>(ga, T, D, smem);
     }
-    const float* res1 = (pre || l == 0) ? B.ra : B.xa;
-    g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
-    g.kdst = kc; g.vdst = vc; g.slot0 = pos0;
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
-
-    attn_phase<W>(D, B.q, kc, vc, B.att, M, pos0, 0, scratch);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
-
-    g = GemmArgs<W>{};
-    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
-    g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
-
-    g = GemmArgs<W>{};
-    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.rb;
-    if (pre) { g.ln_b_g = L.ln2g; g.ln_b_b = L.ln2b; }
-    else { g.ln_a_g = L.ln1g; g.ln_a_b = L.ln1b; g.x_store = B.xb; }
-    const float* res2 = pre ? B.rb : B.xb;
-    g.w = L.wqc; g.bias = L.bqc; g.epi = EPI_STORE; g.out = B.q; g.ld = D.d;
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
-
-    attn_phase<W>(D, B.q, kx, vx, B.att, M, -1, P.n_src, scratch);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
-
-    g = GemmArgs<W>{};
-    g.M = M; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.woc; g.bias = L.boc;
-    g.epi = EPI_RESID; g.out = B.rc; g.ld = D.d; g.resid = res2;
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
-
-    g = GemmArgs<W>{};
-    g.M = M; g.N = D.f; g.K = D.d; g.x_src = B.rc;
-    if (pre) { g.ln_b_g = L.ln3g; g.ln_b_b = L.ln3b; }
-    else { g.ln_a_g = L.ln2g; g.ln_a_b = L.ln2b; g.x_store = B.xc; }
-    const float* res3 = pre ? B.rc : B.xc;
-    g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
-
-    g = GemmArgs<W>{};
-    g.M = M; g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
-    g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res3;
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return false;
+    if (ph == nph - 1) break;            // the LM head ends at the caller's commit barrier
+    const int next = is_attn_phase(ph + 1, nph) ? ph + 2 : ph + 1;
+    if (!grid_barrier(B.bar, tgt, status, [&] {
+          if (!attn && threadIdx.x == 32) gemm_args(P, next, M, pos0, tok, logits, ga);
+          prefetch_phase(P, ph + 3);
+        }))
+      return false;
   }
   return true;
-}
-
-// LM head over the final hidden rows: argmax partials (or raw logits).
-template <typename W>
-__device__ void lm_head(const KParams<W>& P, int M, unsigned char* smem, float* logits) {
-  const Dims& D = P.D;
-  const ModelW<W>& mw = *P.mw;
-  GemmArgs<W> g{};
-  g.M = M; g.N = D.V; g.K = D.d; g.x_src = P.B.ra;
-  g.ln_b_g = D.pre_ln ? mw.dec_lnf_g : mw.dec[D.Ld - 1].ln3g;
-  g.ln_b_b = D.pre_ln ? mw.dec_lnf_b : mw.dec[D.Ld - 1].ln3b;
-  g.w = mw.embed;
-  if (logits != nullptr) { g.epi = EPI_LOGITS; g.out = logits; g.ld = D.V; }
-  else { g.epi = EPI_ARGMAX; g.part = P.B.part; g.part_ld = D.rows; }
-  gemm_phase<W>(g, embed_tabs(P), D, smem);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -341,10 +391,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
   int* status = &B.st->status;
+  load_smem_mw(P);
+#ifdef PD_TIMELINE
+  if (threadIdx.x == 0) { s_tl_n = 0; s_tl_first = g_tl_first; }
+  for (int i = threadIdx.x; i < kTlN * 8; i += blockDim.x) s_tl[i / 8][i % 8] = 0;
+  __syncthreads();
+#endif
 
   if (P.debug_len > 0) {
-    if (!decoder_pass<W>(P, P.debug_len, 0, B.dbg_tok, tgt, smem)) return;
-    lm_head<W>(P, P.debug_len, smem, P.logits);
+    run_pass<W>(P, P.debug_len, 0, B.dbg_tok, P.logits, tgt, smem);
     return;
   }
 
@@ -374,14 +429,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
     __syncthreads();
     if (s_done) break;
     const int M = s_blk, pos0 = s_i - 1;
-    prefetch_pass<W>(P);
     // row r's input is the token at position i-1+r: y_{i-1}, then the block's draft
     // (the shift-left of Algorithm 2's appendix note)
-    if (!decoder_pass<W>(P, M, pos0, B.y + pos0, tgt, smem)) break;
-    lm_head<W>(P, M, smem, nullptr);
+    if (!run_pass<W>(P, M, pos0, B.y + pos0, nullptr, tgt, smem)) break;
     // the last CTA to finish its LM-head columns merges the argmax partials and commits
     if (!grid_barrier_last(B.bar, tgt, status, [&] { commit<W>(P, smem); })) break;
   }
+#ifdef PD_TIMELINE
+  tl_dump();
+#endif
   if (blockIdx.x == 0) {
     __syncthreads();
     write_outputs(P);
@@ -394,7 +450,8 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
   unsigned tgt = 0;
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
-  const ModelW<W>& mw = *P.mw;
+  load_smem_mw(P);
+  const ModelW<W>& mw = smem_mw<W>();
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
@@ -1015,6 +1072,15 @@ void* pd_stream(pd_ctx* c) { return c ? (void*)c->stream : nullptr; }
 int pd_debug_set_prof(void* dptr, int cap) {
   if (cudaMemcpyToSymbol(pd::g_prof, &dptr, sizeof(dptr)) != cudaSuccess) return -3;
   if (cudaMemcpyToSymbol(pd::g_prof_cap, &cap, sizeof(cap)) != cudaSuccess) return -3;
+  return 0;
+}
+#endif
+
+#ifdef PD_TIMELINE
+// Development builds only: record the per-CTA timeline of barrier intervals first..first+51.
+int pd_debug_set_tl(void* dptr, int first) {
+  if (cudaMemcpyToSymbol(pd::g_tl, &dptr, sizeof(dptr)) != cudaSuccess) return -3;
+  if (cudaMemcpyToSymbol(pd::g_tl_first, &first, sizeof(first)) != cudaSuccess) return -3;
   return 0;
 }
 #endif

@@ -165,6 +165,39 @@ __device__ __forceinline__ float act_fn(float v, int act) {
 // grid barriers with bounded waits
 // ------------------------------------------------------------------------------------------
 
+#ifdef PD_TIMELINE
+// Development-only timeline: per-CTA clock marks of kTlN consecutive barrier intervals,
+// held in shared memory while the kernel runs and written out at its end.
+constexpr int kTlN = 52;
+__device__ unsigned long long* g_tl = nullptr;   // [kTlN][grid][8]
+__device__ int g_tl_first = 0;
+__shared__ int s_tl_n, s_tl_first;
+__shared__ unsigned long long s_tl[kTlN][8];
+__device__ __forceinline__ void tl_mark(int k, bool gt) {
+  if (threadIdx.x == 0) {
+    const int i = s_tl_n - s_tl_first;
+    if ((unsigned)i < (unsigned)kTlN) {
+      unsigned long long v;
+      if (gt) { asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(v)); }
+      else { v = clock64(); }
+      s_tl[i][k] = v;
+    }
+  }
+}
+__device__ __forceinline__ void tl_dump() {
+  if (threadIdx.x == 0 && g_tl != nullptr)
+    for (int i = 0; i < kTlN; ++i)
+      for (int k = 0; k < 8; ++k) g_tl[((size_t)i * gridDim.x + blockIdx.x) * 8 + k] = s_tl[i][k];
+}
+#define TL(k) tl_mark(k, false)
+#define TLG(k) tl_mark(k, true)
+#define TL_NEXT() do { if (threadIdx.x == 0) ++s_tl_n; } while (0)
+#else
+#define TL(k) do { } while (0)
+#define TLG(k) do { } while (0)
+#define TL_NEXT() do { } while (0)
+#endif
+
 #ifdef PD_PHASE_TIMING
 // Development-only phase timer: last arrival and release time of every barrier.
 __device__ unsigned long long* g_prof = nullptr;
@@ -219,18 +252,30 @@ __device__ __forceinline__ int spin_until(unsigned* bar, const unsigned* word, u
 // acquire at GPU scope: the bar.sync before the release-add orders every thread's writes of
 // this CTA before the arrival; the acquire load plus the bar.sync after it order the other
 // CTAs' writes before every thread's later reads.  Returns false on abort.
-__device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, int* status) {
+// `during()` runs on every thread between this CTA's arrival and its wait (work that does not
+// depend on the other CTAs, such as preparing the next phase).
+template <typename F>
+__device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, int* status,
+                                             F&& during) {
   __shared__ int s_ok;
   __syncthreads();
   target += gridDim.x;
+  TL(3); TLG(5);
   if (threadIdx.x == 0) {
     PD_PROF_ARRIVE(target);
     red_release_add(bar, 1u);
+  }
+  during();
+  if (threadIdx.x == 0) {
     s_ok = spin_until(bar, bar, target, status);
     PD_PROF_RELEASE(target);
   }
+  TL_NEXT(); TL(0); TLG(4);
   __syncthreads();
   return s_ok != 0;
+}
+__device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, int* status) {
+  return grid_barrier(bar, target, status, [] {});
 }
 
 // A barrier whose last arriving CTA runs `last()` before anybody is released: it sees every
@@ -242,6 +287,7 @@ __device__ __forceinline__ bool grid_barrier_last(unsigned* bar, unsigned& targe
   __shared__ int s_ok, s_last;
   __syncthreads();
   target += gridDim.x;
+  TL(3); TLG(5);
   if (threadIdx.x == 0) {
     PD_PROF_ARRIVE(target);
     const unsigned old = atom_acq_rel_add(bar, 1u);
@@ -257,6 +303,7 @@ __device__ __forceinline__ bool grid_barrier_last(unsigned* bar, unsigned& targe
     s_ok = spin_until(bar, bar + 2, target, status);
   }
   if (threadIdx.x == 0) PD_PROF_RELEASE(target);
+  TL_NEXT(); TL(0); TLG(4);
   __syncthreads();
   return s_ok != 0;
 }
@@ -419,6 +466,14 @@ __device__ __forceinline__ float dot_part(const float* __restrict__ w, int K, in
 }
 
 constexpr int kMaxRowRegs = 8;      // embedded / normalised rows: <= 8 float4 per lane
+constexpr int kStageB = 4;
+__device__ __forceinline__ float4 ld_act4(const float* p) {
+  float4 v;
+  asm volatile("ld.global.cg.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p));
+  return v;
+}
 
 // LayerNorm of a row held as float4 v[i] = elements lane*4 + 128*i: mean and biased variance
 // from per-lane sums in ascending i, then fixed butterflies.
@@ -475,18 +530,34 @@ __device__ void stage_x(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims&
   const int warp = threadIdx.x >> 5;
   const int K = g.K;
   const bool any_ln = g.ln_a_g != nullptr || g.ln_b_g != nullptr || g.emb_tok != nullptr;
+  if (!any_ln) {                         // plain copy (any K multiple of 128), all threads
+    const bool store = g.x_store != nullptr && blockIdx.x == 0;
+    const int K4 = K / 4, F = mt * K4;
+    for (int f0 = 0; f0 < F; f0 += kThreads * kStageB) {
+      float4 v[kStageB];
+#pragma unroll
+      for (int j = 0; j < kStageB; ++j) {
+        const int f = f0 + j * kThreads + (int)threadIdx.x;
+        if (f < F) {
+          const int r = f / K4, k = (f - r * K4) * 4;
+          v[j] = ld_act4(g.x_src + (size_t)(m0 + r) * K + k);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < kStageB; ++j) {
+        const int f = f0 + j * kThreads + (int)threadIdx.x;
+        if (f < F) {
+          const int r = f / K4, k = (f - r * K4) * 4;
+          if (store) *reinterpret_cast<float4*>(g.x_store + (size_t)(m0 + r) * K + k) = v[j];
+          put4(xs + (size_t)r * K + k, v[j]);
+        }
+      }
+    }
+    return;
+  }
   for (int r = warp; r < mt; r += kWarps) {
     const int m = m0 + r;
     const bool store = g.x_store != nullptr && blockIdx.x == 0;
-    if (!any_ln) {                       // plain copy (any K multiple of 128)
-      const float* src = g.x_src + (size_t)m * K;
-      for (int k = lane * 4; k < K; k += 128) {
-        const float4 v = *reinterpret_cast<const float4*>(src + k);
-        if (store) *reinterpret_cast<float4*>(g.x_store + (size_t)m * K + k) = v;
-        put4(xs + (size_t)r * K + k, v);
-      }
-      continue;
-    }
     const int nI = K / 128;              // K <= 1024 for rows that are embedded or normalised
     float4 v[kMaxRowRegs];
     if (g.emb_tok != nullptr) {
@@ -595,9 +666,12 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
   const int c = lane / kMTile, r = lane % kMTile;   // the (column, row) this lane finishes
   for (int m0 = 0; m0 < g.M; m0 += kMTile) {
     const int mt = g.M - m0 < kMTile ? g.M - m0 : kMTile;
+    if (m0 == 0) TL(6);
     __syncthreads();
     stage_x(g, T, D, m0, mt, xs);
+    if (m0 == 0) TL(7);
     __syncthreads();
+    if (m0 == 0) TL(1);
     float amx = -INFINITY, asum = 0.f;
     int aidx = 0x7fffffff, anan = 0;
     for (int base = 0; base < ngroups; base += stride) {
@@ -645,6 +719,7 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
         case EPI_LOGITS: g.out[(size_t)m * g.ld + n] = v; break;
       }
     }
+    if (m0 == 0) TL(2);
     if (g.epi == EPI_ARGMAX) {
       // lane c*kMTile + r of a part-0 warp holds row r over its columns n0 + c: merge in warp
       // order, then lane (column) order, and publish the CTA partial per row
