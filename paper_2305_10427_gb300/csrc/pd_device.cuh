@@ -234,10 +234,13 @@ __device__ __forceinline__ void st_release_u32(unsigned* p, unsigned v) {
 // Bar words: [0] arrival counter (only grows), [1] abort flag, [2] release word of the
 // commit barrier.  Spin until *word >= target; give up after kWaitNs, raising the abort flag
 // and PD_ETIMEOUT, so that a broken schedule ends the kernel instead of hanging the GPU.
+// The abort flag and the clock are looked at every 32nd poll only: a poll is then a single
+// load, and the barrier is released one round trip after its last arrival.
 __device__ __forceinline__ int spin_until(unsigned* bar, const unsigned* word, unsigned target,
                                           int* status) {
   const unsigned long long t0 = globaltimer_ns();
-  while (ld_acquire_u32(word) < target) {
+  for (unsigned n = 1; ld_acquire_u32(word) < target; ++n) {
+    if ((n & 31u) != 0u) continue;
     if (ld_acquire_u32(bar + 1) != 0u) return 0;
     if (globaltimer_ns() - t0 > kWaitNs) {
       atomicExch(bar + 1, 1u);
