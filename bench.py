@@ -34,8 +34,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
 # ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel sources whose
 # SHA-256 is recorded here; any other source reports traffic null.
-DRAM_BYTES_PER_PASS = 29.9e6
-DRAM_SOURCES_SHA256 = "857e8c5220d4ea0b167edfa0f80eedc3ad47a89e093c3e11693301a45fa630e8"
+DRAM_BYTES_PER_PASS = 12.35e6
+DRAM_SOURCES_SHA256 = "1c67fbc3847d050d0d94cdb2b2d4c27c3a842849fd7cb732f01fc67baf8b5ea9"
 
 
 def kernel_sources_sha256() -> str:

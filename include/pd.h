@@ -156,6 +156,15 @@ pd_status pd_debug_logits(pd_ctx* ctx, const int32_t* y_in, int len, float* logi
  * Synchronous; calls no device allocator. */
 pd_status pd_debug_logits_static(pd_ctx* ctx, const int32_t* y_in, int len, float* logits);
 
+/* Test-only failure-detection check (the paper has no counterpart).  Runs, on the context's
+ * stream, one thread of the kernels' bounded device-side wait (the wait of the grid barriers)
+ * against a counter that nothing advances, with a limit of limit_ns nanoseconds instead of the
+ * kernels' 10 s.  The wait must give up: on return *status holds the status the device raised
+ * (PD_ETIMEOUT expected), and the call returns PD_OK if the wait also raised its abort flag
+ * (PD_ESTATE otherwise).  limit_ns in (0, 1e10]; PD_EINVAL otherwise.  Synchronous; allocates
+ * and frees 16 bytes of device memory; the context stays usable. */
+pd_status pd_debug_wait_timeout(pd_ctx* ctx, uint64_t limit_ns, int* status);
+
 /* The context's cudaStream_t. */
 void* pd_stream(pd_ctx* ctx);
 

@@ -26,8 +26,8 @@ METHODS = {"greedy": 0, "jacobi": 1, "gs_jacobi": 2, "hybrid_gs_jacobi": 3}
 # Every symbol include/pd.h declares.
 EXPORTED = ("pd_weights_nbytes", "pd_create", "pd_export_weights", "pd_encode",
             "pd_encode_device", "pd_decode", "pd_decode_device", "pd_debug_logits",
-            "pd_debug_logits_static", "pd_stream", "pd_launch_count", "pd_last_error",
-            "pd_destroy")
+            "pd_debug_logits_static", "pd_debug_wait_timeout", "pd_stream", "pd_launch_count",
+            "pd_last_error", "pd_destroy")
 
 
 class PdError(RuntimeError):
@@ -89,6 +89,8 @@ def load_library() -> ctypes.CDLL:
     lib.pd_debug_logits.restype = I
     lib.pd_debug_logits_static.argtypes = [P, pi32, I, ctypes.POINTER(ctypes.c_float)]
     lib.pd_debug_logits_static.restype = I
+    lib.pd_debug_wait_timeout.argtypes = [P, ctypes.c_uint64, pint]
+    lib.pd_debug_wait_timeout.restype = I
     lib.pd_stream.argtypes = [P]
     lib.pd_stream.restype = P
     lib.pd_launch_count.argtypes = [P]
@@ -242,6 +244,14 @@ class Decoder:
             self._h, _i32p(a), int(a.size), out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))),
             "pd_debug_logits_static")
         return out
+
+    def debug_wait_timeout(self, limit_ns: int) -> int:
+        """Run the device wait against a counter nothing advances, limited to limit_ns; returns
+        the status the device raised (PD_ETIMEOUT expected)."""
+        st = ctypes.c_int(0)
+        self._check(self._lib.pd_debug_wait_timeout(self._h, ctypes.c_uint64(int(limit_ns)),
+                                                    ctypes.byref(st)), "pd_debug_wait_timeout")
+        return int(st.value)
 
     def export_weights(self, dtype) -> np.ndarray:
         out = np.zeros(self.blob_nbytes // np.dtype(dtype).itemsize, dtype=dtype)

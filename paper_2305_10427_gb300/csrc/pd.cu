@@ -1065,16 +1065,32 @@ pd_status pd_debug_logits_static(pd_ctx* c, const int32_t* y_in, int len, float*
   return PD_OK;
 }
 
-void* pd_stream(pd_ctx* c) { return c ? (void*)c->stream : nullptr; }
-
-#ifdef PD_PHASE_TIMING
-// Development builds only: point the device phase timer at a buffer of 2 * cap uint64.
-int pd_debug_set_prof(void* dptr, int cap) {
-  if (cudaMemcpyToSymbol(pd::g_prof, &dptr, sizeof(dptr)) != cudaSuccess) return -3;
-  if (cudaMemcpyToSymbol(pd::g_prof_cap, &cap, sizeof(cap)) != cudaSuccess) return -3;
-  return 0;
+pd_status pd_debug_wait_timeout(pd_ctx* c, uint64_t limit_ns, int* status) {
+  if (!c) return PD_EINVAL;
+  if (!status || limit_ns == 0 || limit_ns > 10000000000ull)
+    return fail(c, PD_EINVAL, "limit_ns must be in (0, 1e10] and status non-NULL");
+  unsigned* words = nullptr;   // [0] counter, [1] abort flag, [2] unused, [3] the status
+  PD_CUDA(c, cudaMalloc(&words, 4 * sizeof(unsigned)));
+  pd_status st = PD_OK;
+  int host[4] = {0, 0, 0, 0};
+  if (cudaMemsetAsync(words, 0, 4 * sizeof(unsigned), c->stream) != cudaSuccess) st = PD_ECUDA;
+  if (st == PD_OK) {
+    pd::wait_probe_kernel<<<1, 32, 0, c->stream>>>(words, reinterpret_cast<int*>(words + 3),
+                                                   (unsigned long long)limit_ns);
+    c->launches += 1;
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemcpyAsync(host, words, sizeof(host), cudaMemcpyDeviceToHost, c->stream) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(c->stream) != cudaSuccess)
+      st = PD_ECUDA;
+  }
+  cudaFree(words);
+  if (st != PD_OK) return fail(c, st, "wait probe failed");
+  *status = host[3];
+  return host[1] != 0u ? PD_OK : fail(c, PD_ESTATE, "the probe's abort flag was not raised");
 }
-#endif
+
+void* pd_stream(pd_ctx* c) { return c ? (void*)c->stream : nullptr; }
 
 #ifdef PD_TIMELINE
 // Development builds only: record the per-CTA timeline of barrier intervals first..first+51.

@@ -166,8 +166,11 @@ __device__ __forceinline__ float act_fn(float v, int act) {
 // ------------------------------------------------------------------------------------------
 
 #ifdef PD_TIMELINE
-// Development-only timeline: per-CTA clock marks of kTlN consecutive barrier intervals,
-// held in shared memory while the kernel runs and written out at its end.
+// Development-only timeline: per-CTA clock marks of kTlN consecutive barrier intervals (from
+// interval g_tl_first on), held in shared memory while the kernel runs and written out at its
+// end.  Marks of an interval: 0 / 4 release of the barrier that opens it (clock64 /
+// globaltimer), 6 GEMM tile start, 7 this warp's rows staged, 1 all rows staged, 2 tile
+// products and epilogue done, 3 / 5 arrival at the barrier that closes it.
 constexpr int kTlN = 52;
 __device__ unsigned long long* g_tl = nullptr;   // [kTlN][grid][8]
 __device__ int g_tl_first = 0;
@@ -198,25 +201,6 @@ __device__ __forceinline__ void tl_dump() {
 #define TL_NEXT() do { } while (0)
 #endif
 
-#ifdef PD_PHASE_TIMING
-// Development-only phase timer: last arrival and release time of every barrier.
-__device__ unsigned long long* g_prof = nullptr;
-__device__ int g_prof_cap = 0;
-#define PD_PROF_ARRIVE(target)                                                             \
-  do {                                                                                     \
-    const int pidx_ = (int)((target) / gridDim.x);                                         \
-    if (g_prof != nullptr && pidx_ < g_prof_cap) atomicMax(&g_prof[2 * pidx_], globaltimer_ns()); \
-  } while (0)
-#define PD_PROF_RELEASE(target)                                                            \
-  do {                                                                                     \
-    const int pidx_ = (int)((target) / gridDim.x);                                         \
-    if (g_prof != nullptr && pidx_ < g_prof_cap && blockIdx.x == 0)                        \
-      g_prof[2 * pidx_ + 1] = globaltimer_ns();                                            \
-  } while (0)
-#else
-#define PD_PROF_ARRIVE(target) do { } while (0)
-#define PD_PROF_RELEASE(target) do { } while (0)
-#endif
 
 __device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
@@ -237,18 +221,26 @@ __device__ __forceinline__ void st_release_u32(unsigned* p, unsigned v) {
 // The abort flag and the clock are looked at every 32nd poll only: a poll is then a single
 // load, and the barrier is released one round trip after its last arrival.
 __device__ __forceinline__ int spin_until(unsigned* bar, const unsigned* word, unsigned target,
-                                          int* status) {
+                                          int* status,
+                                          unsigned long long limit_ns = kWaitNs) {
   const unsigned long long t0 = globaltimer_ns();
   for (unsigned n = 1; ld_acquire_u32(word) < target; ++n) {
     if ((n & 31u) != 0u) continue;
     if (ld_acquire_u32(bar + 1) != 0u) return 0;
-    if (globaltimer_ns() - t0 > kWaitNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
       atomicExch(bar + 1, 1u);
       atomicCAS(status, 0, (int)PD_ETIMEOUT);
       return 0;
     }
   }
   return 1;
+}
+
+// Failure-detection check: one thread waits, with the barrier's bounded wait, for a counter
+// that nothing advances (bar[0] stays 0, target 1).  The wait must give up after limit_ns,
+// raise the abort flag and PD_ETIMEOUT in *status, and return.
+__global__ void wait_probe_kernel(unsigned* bar, int* status, unsigned long long limit_ns) {
+  if (blockIdx.x == 0 && threadIdx.x == 0) (void)spin_until(bar, bar, 1u, status, limit_ns);
 }
 
 // All CTAs of the (cooperatively launched, hence co-resident) grid meet here.  Release /
@@ -265,13 +257,11 @@ __device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, in
   target += gridDim.x;
   TL(3); TLG(5);
   if (threadIdx.x == 0) {
-    PD_PROF_ARRIVE(target);
     red_release_add(bar, 1u);
   }
   during();
   if (threadIdx.x == 0) {
     s_ok = spin_until(bar, bar, target, status);
-    PD_PROF_RELEASE(target);
   }
   TL_NEXT(); TL(0); TLG(4);
   __syncthreads();
@@ -292,7 +282,6 @@ __device__ __forceinline__ bool grid_barrier_last(unsigned* bar, unsigned& targe
   target += gridDim.x;
   TL(3); TLG(5);
   if (threadIdx.x == 0) {
-    PD_PROF_ARRIVE(target);
     const unsigned old = atom_acq_rel_add(bar, 1u);
     s_last = old + 1u == target;
     s_ok = 1;
@@ -305,7 +294,6 @@ __device__ __forceinline__ bool grid_barrier_last(unsigned* bar, unsigned& targe
   } else if (threadIdx.x == 0) {
     s_ok = spin_until(bar, bar + 2, target, status);
   }
-  if (threadIdx.x == 0) PD_PROF_RELEASE(target);
   TL_NEXT(); TL(0); TLG(4);
   __syncthreads();
   return s_ok != 0;

@@ -73,6 +73,7 @@ def test_wrong_blob_size_is_rejected(lib):
 def test_null_context_calls(lib):
     assert lib.pd_encode(None, None, 3) == B.PD_EINVAL
     assert lib.pd_decode_device(None, None, None, None) == B.PD_EINVAL
+    assert lib.pd_debug_wait_timeout(None, 1000, None) == B.PD_EINVAL
     assert lib.pd_launch_count(None) == 0
     assert lib.pd_last_error(None) == b"context is NULL"
     lib.pd_destroy(None)
