@@ -13,6 +13,7 @@ Multi-GPU: replicas (every rank decodes the full sentence set; weak scaling).
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -389,9 +390,13 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="marian", choices=["marian", "marian-knob"],
+    ap.add_argument("--workload", default="marian", choices=["marian", "marian-knob", "mbart"],
                     help="marian: the benchmark workload; marian-knob: the same model with a "
-                         "small token-embedding scale (Jacobi accepts several tokens per pass)")
+                         "small token-embedding scale (Jacobi accepts several tokens per pass); "
+                         "mbart: the mBART-large-sized model (pre-LN, GELU, learned positions, "
+                         "V = 250027), 128 sentences of 16..128 ids")
+    ap.add_argument("--b", type=int, default=0,
+                    help="GS-Jacobi block size (default: the workload's, 5)")
     ap.add_argument("--all-methods", action="store_true",
                     help="also time full-sentence Jacobi and Hybrid GS-Jacobi (b=3), one step each")
     ap.add_argument("--sentences", type=int, default=0,
@@ -400,6 +405,11 @@ def main():
     global WORKLOAD
     if args.workload == "marian-knob":
         WORKLOAD = synth.MARIAN_KNOB
+    elif args.workload == "mbart":
+        WORKLOAD = synth.MBART_GS
+    if args.b and args.b != WORKLOAD.b:
+        WORKLOAD = dataclasses.replace(
+            WORKLOAD, b=args.b, name=WORKLOAD.name.replace(f"b={WORKLOAD.b}", f"b={args.b}"))
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

@@ -417,3 +417,25 @@ def test_pre_ln_models(name, request):
         compared += compare_with_oracle_runs(s, src, max_len, res)
     if s.spec.dtype == synth.DTYPE_F32:
         assert compared >= 3
+
+
+def test_mbart_full_size_sampled():
+    """The mBART-large-sized preset at its full size (d = 1024, 12 + 12 layers, d_ff = 4096,
+    V = 250027, pre-LN, GELU, learned positions): teacher-forced logits of a few rows against
+    the oracle, and GS-Jacobi b = 5 / b = 16 equal to greedy with the tokens checked by one
+    teacher-forced oracle pass (sampled outputs: the oracle runs the model at full size)."""
+    s = Setup(synth.MBART, 16, 16, seed=0)
+    rng = np.random.default_rng(31)
+    src = synth.MBART_GS.sentences()[0][:10]
+    s.dec.encode(src)
+    y_in = np.r_[synth.BOS_ID, rng.integers(3, s.spec.vocab, size=3)].astype(np.int32)
+    got = s.dec.debug_logits(y_in)
+    assert rel_row_err(got, s.model.logits(s.mem(src), y_in)).max() < 2e-2
+    s.dec.encode(src)
+    g = s.dec.decode("greedy", 12)
+    for b in (5, 16):
+        r = s.dec.decode("gs_jacobi", 12, b=b)
+        assert r.tokens == g.tokens, b
+        assert r.n_iters <= 12
+    check_tokens_teacher_forced(s, src, g.tokens)
+    s.dec.close()
