@@ -38,8 +38,15 @@ struct KParams {
 };
 
 struct SmemLayout {
-  size_t xs, part, scratch, commit, total;
+  size_t xs, part, scratch, commit, ln, ln_bytes, total;
 };
+
+// The decoder's LayerNorm vectors (per layer ln1, ln2, ln3 gamma / beta, and the embedding and
+// final LayerNorms of pre-LN models), kept in shared memory when they fit in kLnSmemMax bytes.
+constexpr size_t kLnSmemMax = 64 * 1024;
+__host__ __device__ inline size_t ln_vectors(const Dims& D) {
+  return (size_t)D.Ld * 6 + (D.pre_ln ? 4 : 0);
+}
 
 __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   SmemLayout L;
@@ -48,7 +55,10 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   L.part = L.xs + ((size_t)kMTile * kmax * wsize + 15) / 16 * 16;
   L.scratch = L.part + (size_t)kWarps * 32 * sizeof(Partial);
   L.commit = L.scratch + (size_t)kWarps * (128 + D.rows + 4) * sizeof(float);
-  L.total = L.commit + (size_t)(D.max_tgt + 1) * 3 * sizeof(int) + 64;
+  L.ln = (L.commit + (size_t)(D.max_tgt + 1) * 3 * sizeof(int) + 64 + 15) / 16 * 16;
+  const size_t lnb = ln_vectors(D) * D.d * wsize;
+  L.ln_bytes = lnb <= kLnSmemMax ? lnb : 0;
+  L.total = L.ln + L.ln_bytes;
   return L;
 }
 
@@ -70,6 +80,50 @@ __device__ __forceinline__ void load_smem_mw(const KParams<W>& P) {
   const unsigned long long* src = reinterpret_cast<const unsigned long long*>(P.mw);
   unsigned long long* dst = reinterpret_cast<unsigned long long*>(&smem_mw<W>());
   for (int i = threadIdx.x; i < (int)(sizeof(ModelW<W>) / 8); i += blockDim.x) dst[i] = src[i];
+  __syncthreads();
+}
+
+// Copy the decoder's LayerNorm vectors into the shared-memory region (when the layout has
+// one) and point the shared pointer table at the copies: a LayerNorm prologue then reads its
+// gamma / beta from shared memory instead of making an L2 round trip after the statistics.
+template <typename W>
+__device__ void load_smem_ln(const Dims& D, unsigned char* smem) {
+  const SmemLayout L = smem_layout(D, sizeof(W));
+  if (L.ln_bytes == 0) return;
+  ModelW<W>& mw = smem_mw<W>();
+  W* dst = reinterpret_cast<W*>(smem + L.ln);
+  const int nv = (int)ln_vectors(D);
+  const int chunks = D.d * (int)sizeof(W) / 16;            // 16-byte pieces per vector
+  auto vec = [&](int v) -> const W*& {
+    if (v < 6 * D.Ld) {
+      DecLayerW<W>& Ly = mw.dec[v / 6];
+      switch (v % 6) {
+        case 0: return Ly.ln1g;
+        case 1: return Ly.ln1b;
+        case 2: return Ly.ln2g;
+        case 3: return Ly.ln2b;
+        case 4: return Ly.ln3g;
+        default: return Ly.ln3b;
+      }
+    }
+    switch (v - 6 * D.Ld) {
+      case 0: return mw.dec_lne_g;
+      case 1: return mw.dec_lne_b;
+      case 2: return mw.dec_lnf_g;
+      default: return mw.dec_lnf_b;
+    }
+  };
+  for (int i = threadIdx.x; i < nv * chunks; i += blockDim.x) {
+    const int v = i / chunks, j = i - v * chunks;
+    const W* src = vec(v);
+    if (src != nullptr)
+      *reinterpret_cast<uint4*>(reinterpret_cast<char*>(dst + (size_t)v * D.d) + j * 16) =
+          ldg_nc_v4(reinterpret_cast<const char*>(src) + j * 16);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0)
+    for (int v = 0; v < nv; ++v)
+      if (vec(v) != nullptr) vec(v) = dst + (size_t)v * D.d;
   __syncthreads();
 }
 
@@ -392,6 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   const Bufs<W>& B = P.B;
   int* status = &B.st->status;
   load_smem_mw(P);
+  load_smem_ln<W>(D, smem);
 #ifdef PD_TIMELINE
   if (threadIdx.x == 0) { s_tl_n = 0; s_tl_first = g_tl_first; }
   for (int i = threadIdx.x; i < kTlN * 8; i += blockDim.x) s_tl[i / 8][i % 8] = 0;
