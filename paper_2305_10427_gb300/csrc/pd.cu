@@ -41,11 +41,20 @@ struct SmemLayout {
   size_t xs, part, scratch, commit, ln, ln_bytes, total;
 };
 
-// The decoder's LayerNorm vectors (per layer ln1, ln2, ln3 gamma / beta, and the embedding and
-// final LayerNorms of pre-LN models), kept in shared memory when they fit in kLnSmemMax bytes.
-constexpr size_t kLnSmemMax = 64 * 1024;
-__host__ __device__ inline size_t ln_vectors(const Dims& D) {
-  return (size_t)D.Ld * 6 + (D.pre_ln ? 4 : 0);
+// The decoder's small vectors kept in shared memory: the LayerNorm vectors (per layer ln1,
+// ln2, ln3 gamma / beta, and the embedding and final LayerNorms of pre-LN models) when they fit
+// in kVecSmemMax bytes, and with them the biases (per layer qkv, o, cross-q, cross-o, ffn1,
+// ffn2) when both fit.  Per layer, in elements: 6 d of LayerNorm, then 7 d + f of bias.
+constexpr size_t kVecSmemMax = 112 * 1024;
+__host__ __device__ inline size_t ln_elems(const Dims& D) {
+  return ((size_t)D.Ld * 6 + (D.pre_ln ? 4 : 0)) * D.d;
+}
+__host__ __device__ inline size_t bias_elems(const Dims& D) {
+  return (size_t)D.Ld * (7 * (size_t)D.d + D.f);
+}
+__host__ __device__ inline size_t vec_smem_bytes(const Dims& D, size_t wsize) {
+  const size_t ln = ln_elems(D) * wsize, all = ln + bias_elems(D) * wsize;
+  return all <= kVecSmemMax ? all : (ln <= kVecSmemMax ? ln : 0);
 }
 
 __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
@@ -56,8 +65,7 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   L.scratch = L.part + (size_t)kWarps * 32 * sizeof(Partial);
   L.commit = L.scratch + (size_t)kWarps * (128 + D.rows + 4) * sizeof(float);
   L.ln = (L.commit + (size_t)(D.max_tgt + 1) * 3 * sizeof(int) + 64 + 15) / 16 * 16;
-  const size_t lnb = ln_vectors(D) * D.d * wsize;
-  L.ln_bytes = lnb <= kLnSmemMax ? lnb : 0;
+  L.ln_bytes = vec_smem_bytes(D, wsize);
   L.total = L.ln + L.ln_bytes;
   return L;
 }
@@ -83,18 +91,23 @@ __device__ __forceinline__ void load_smem_mw(const KParams<W>& P) {
   __syncthreads();
 }
 
-// Copy the decoder's LayerNorm vectors into the shared-memory region (when the layout has
-// one) and point the shared pointer table at the copies: a LayerNorm prologue then reads its
-// gamma / beta from shared memory instead of making an L2 round trip after the statistics.
+// Copy the decoder's LayerNorm vectors (and biases, see vec_smem_bytes) into the shared-memory
+// region and point the shared pointer table at the copies: a LayerNorm prologue then reads its
+// gamma / beta, and an epilogue its bias, from shared memory instead of making an L2 round
+// trip (every barrier's acquire drops the SM's L1 copies of global data).
 template <typename W>
-__device__ void load_smem_ln(const Dims& D, unsigned char* smem) {
+__device__ void load_smem_vectors(const Dims& D, unsigned char* smem) {
   const SmemLayout L = smem_layout(D, sizeof(W));
   if (L.ln_bytes == 0) return;
+  const bool with_bias = L.ln_bytes > ln_elems(D) * sizeof(W);
   ModelW<W>& mw = smem_mw<W>();
   W* dst = reinterpret_cast<W*>(smem + L.ln);
-  const int nv = (int)ln_vectors(D);
-  const int chunks = D.d * (int)sizeof(W) / 16;            // 16-byte pieces per vector
-  auto vec = [&](int v) -> const W*& {
+  // vector v: its pointer field in the shared table and its length (elements); laid out in
+  // order, LayerNorm vectors first
+  const int nln = 6 * D.Ld + (D.pre_ln ? 4 : 0);
+  const int nv = nln + (with_bias ? 6 * D.Ld : 0);
+  auto field = [&](int v, int& len) -> const W*& {
+    len = D.d;
     if (v < 6 * D.Ld) {
       DecLayerW<W>& Ly = mw.dec[v / 6];
       switch (v % 6) {
@@ -106,24 +119,48 @@ __device__ void load_smem_ln(const Dims& D, unsigned char* smem) {
         default: return Ly.ln3b;
       }
     }
-    switch (v - 6 * D.Ld) {
-      case 0: return mw.dec_lne_g;
-      case 1: return mw.dec_lne_b;
-      case 2: return mw.dec_lnf_g;
-      default: return mw.dec_lnf_b;
+    if (v < nln) {
+      switch (v - 6 * D.Ld) {
+        case 0: return mw.dec_lne_g;
+        case 1: return mw.dec_lne_b;
+        case 2: return mw.dec_lnf_g;
+        default: return mw.dec_lnf_b;
+      }
+    }
+    DecLayerW<W>& Ly = mw.dec[(v - nln) / 6];
+    switch ((v - nln) % 6) {
+      case 0: len = 3 * D.d; return Ly.bqkv;
+      case 1: return Ly.bo;
+      case 2: return Ly.bqc;
+      case 3: return Ly.boc;
+      case 4: len = D.f; return Ly.b1;
+      default: return Ly.b2;
     }
   };
-  for (int i = threadIdx.x; i < nv * chunks; i += blockDim.x) {
-    const int v = i / chunks, j = i - v * chunks;
-    const W* src = vec(v);
-    if (src != nullptr)
-      *reinterpret_cast<uint4*>(reinterpret_cast<char*>(dst + (size_t)v * D.d) + j * 16) =
-          ldg_nc_v4(reinterpret_cast<const char*>(src) + j * 16);
+  // every warp copies vectors v = warp, warp + kWarps, ... (16 bytes per lane and step)
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  size_t off = 0;
+  for (int v = 0; v < nv; ++v) {
+    int len;
+    const W* src = field(v, len);
+    if (v % kWarps == warp && src != nullptr) {
+      const int chunks = len * (int)sizeof(W) / 16;
+      for (int j = lane; j < chunks; j += 32)
+        *reinterpret_cast<uint4*>(reinterpret_cast<char*>(dst + off) + j * 16) =
+            ldg_nc_v4(reinterpret_cast<const char*>(src) + j * 16);
+    }
+    off += len;
   }
   __syncthreads();
-  if (threadIdx.x == 0)
-    for (int v = 0; v < nv; ++v)
-      if (vec(v) != nullptr) vec(v) = dst + (size_t)v * D.d;
+  if (threadIdx.x == 0) {
+    off = 0;
+    for (int v = 0; v < nv; ++v) {
+      int len;
+      const W*& f = field(v, len);
+      if (f != nullptr) f = dst + off;
+      off += len;
+    }
+  }
   __syncthreads();
 }
 
@@ -446,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   const Bufs<W>& B = P.B;
   int* status = &B.st->status;
   load_smem_mw(P);
-  load_smem_ln<W>(D, smem);
+  load_smem_vectors<W>(D, smem);
 #ifdef PD_TIMELINE
   if (threadIdx.x == 0) { s_tl_n = 0; s_tl_first = g_tl_first; }
   for (int i = threadIdx.x; i < kTlN * 8; i += blockDim.x) s_tl[i / 8][i % 8] = 0;
