@@ -35,8 +35,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
 # ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel sources whose
 # SHA-256 is recorded here; any other source reports traffic null.
-DRAM_BYTES_PER_PASS = 12.35e6
-DRAM_SOURCES_SHA256 = "1c67fbc3847d050d0d94cdb2b2d4c27c3a842849fd7cb732f01fc67baf8b5ea9"
+DRAM_BYTES_PER_PASS = 12.17e6
+DRAM_SOURCES_SHA256 = "c6f72a38673382cbc013233a9a6706918402159979d2fcb1e4fb47550b82db8e"
 
 
 def kernel_sources_sha256() -> str:
