@@ -199,6 +199,7 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const in
     g.w = mw.embed;
     if (logits != nullptr) { g.epi = EPI_LOGITS; g.out = logits; g.ld = D.V; }
     else { g.epi = EPI_ARGMAX; g.part = B.part; g.part_ld = D.rows; }
+    gemm_plan(g, gridDim.x);
     return;
   }
   const int l = ph >> 3;
@@ -249,6 +250,7 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const in
       g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = pre ? B.rc : B.xc;
       break;
   }
+  gemm_plan(g, gridDim.x);
 }
 
 // Ask L2 for the weight rows this CTA reads in GEMM phase ph (nothing for attention phases),
@@ -324,15 +326,6 @@ __device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, f
 // ------------------------------------------------------------------------------------------
 // fixed-point commit (one CTA): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
 // ------------------------------------------------------------------------------------------
-
-__device__ __forceinline__ Partial shfl_partial(const Partial& a, int o) {
-  Partial b;
-  b.mx = __shfl_xor_sync(0xffffffffu, a.mx, o);
-  b.idx = __shfl_xor_sync(0xffffffffu, a.idx, o);
-  b.sum = __shfl_xor_sync(0xffffffffu, a.sum, o);
-  b.nan = __shfl_xor_sync(0xffffffffu, a.nan, o);
-  return b;
-}
 
 // The decoding state is copied into shared memory with one load per field (issued together),
 // the block's previous draft likewise; one thread then takes the decisions from shared memory
@@ -575,6 +568,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     const float* res1 = (pre || l == 0) ? B.ra : B.xa;
     g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
     g.kdst_f = B.k; g.vdst_f = B.v;
+    gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
@@ -584,6 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     g = GemmArgs<W>{};
     g.M = n; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
     g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
+    gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
@@ -593,12 +588,14 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     else { g.ln_a_g = L.ln1g; g.ln_a_b = L.ln1b; g.x_store = B.xb; }
     const float* res2 = pre ? B.rb : B.xb;
     g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
+    gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
     g = GemmArgs<W>{};
     g.M = n; g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
     g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res2;
+    gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
   }
@@ -611,6 +608,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     g.w = mw.dec[l].wkvc; g.bias = mw.dec[l].bkvc; g.epi = EPI_KVCROSS;
     g.kdst = B.kcross + (size_t)l * D.max_src * D.d;
     g.vdst = B.vcross + (size_t)l * D.max_src * D.d;
+    gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
   }
 }

@@ -347,6 +347,10 @@ struct GemmArgs {
   int slot0;
   Partial* part;            // ARGMAX: [grid][rows_ld]
   int part_ld;
+  // How the phase is divided over the grid (gemm_plan): column groups, K-steps per warp,
+  // warps per group, groups per CTA, groups per round; per warp its group slot and K part.
+  int ngroups, spw, kw, gpc, stride;
+  unsigned char wslot[kWarps], wpart[kWarps];
 };
 
 // Embedding and position tables (read by the GEMM whose input is the embedding).
@@ -616,6 +620,15 @@ __device__ __forceinline__ void argmax_push(float v, int col, float& mx, int& id
   }
 }
 
+__device__ __forceinline__ Partial shfl_partial(const Partial& a, int o) {
+  Partial b;
+  b.mx = __shfl_xor_sync(0xffffffffu, a.mx, o);
+  b.idx = __shfl_xor_sync(0xffffffffu, a.idx, o);
+  b.sum = __shfl_xor_sync(0xffffffffu, a.sum, o);
+  b.nan = __shfl_xor_sync(0xffffffffu, a.nan, o);
+  return b;
+}
+
 // a <- a (+) b: larger max wins, equal maxima keep the lower index; sums rescaled.
 __device__ __forceinline__ void partial_merge(Partial& a, const Partial& b) {
   a.nan |= b.nan;
@@ -628,6 +641,25 @@ __device__ __forceinline__ void partial_merge(Partial& a, const Partial& b) {
   } else {
     a.sum = a.sum + b.sum * expf(b.mx - a.mx);
     if (b.mx == a.mx && b.idx < a.idx) a.idx = b.idx;
+  }
+}
+
+// The division of a GEMM phase over the grid, a function of N, K and the grid only: K-steps
+// per warp are 1 when the phase then still fits in one round over the grid (shorter dot chains
+// for the small GEMMs), else 2.  Computed once per phase by the thread that writes the
+// arguments, off the phase's chain of dependent steps.
+template <typename W>
+__device__ __forceinline__ void gemm_plan(GemmArgs<W>& g, int grid) {
+  const int steps = g.K / KStep<W>::E;
+  g.ngroups = (g.N + kNCol - 1) / kNCol;
+  g.spw = (steps <= kWarps && g.ngroups <= grid * (kWarps / steps)) ? 1 : 2;
+  g.kw = (steps + g.spw - 1) / g.spw;
+  g.gpc = kWarps / g.kw;
+  g.stride = grid * g.gpc;
+  for (int w = 0, sl = 0, pt = 0; w < kWarps; ++w) {
+    g.wslot[w] = (unsigned char)sl;
+    g.wpart[w] = (unsigned char)pt;
+    if (++pt == g.kw) { pt = 0; ++sl; }
   }
 }
 
@@ -644,16 +676,10 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
   float* red = reinterpret_cast<float*>(small);           // [kWarps][32] (not used with ps)
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  // K-steps per warp: 1 when the phase then still fits in one round over the grid (shorter
-  // dot chains for the small GEMMs), else 2.  A function of N, K and the grid only.
   const int steps = g.K / KStep<W>::E;
-  const int ngroups = (g.N + kNCol - 1) / kNCol;
-  const int spw = (steps <= kWarps && ngroups <= (int)gridDim.x * (kWarps / steps)) ? 1 : 2;
-  const int kw = (steps + spw - 1) / spw;
-  const int gpc = kWarps / kw;
-  const int slot = warp / kw, part = warp - slot * kw;
+  const int ngroups = g.ngroups, spw = g.spw, kw = g.kw, gpc = g.gpc, stride = g.stride;
+  const int slot = g.wslot[warp], part = g.wpart[warp];
   const int s0 = spw * part, ns = steps - s0 < spw ? steps - s0 : spw;
-  const int stride = gridDim.x * gpc;
   const int c = lane / kMTile, r = lane % kMTile;   // the (column, row) this lane finishes
   for (int m0 = 0; m0 < g.M; m0 += kMTile) {
     const int mt = g.M - m0 < kMTile ? g.M - m0 : kMTile;
@@ -712,17 +738,20 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
     }
     if (m0 == 0) TL(2);
     if (g.epi == EPI_ARGMAX) {
-      // lane c*kMTile + r of a part-0 warp holds row r over its columns n0 + c: merge in warp
-      // order, then lane (column) order, and publish the CTA partial per row
+      // lane c*kMTile + r of a part-0 warp holds row r over its columns n0 + c.  Row r's
+      // kWarps * kNCol partials are merged by warp r: lane l takes entries l, l + 32, ...
+      // (entry e = warp w2, column c2 with e = w2 * kNCol + c2), then a fixed butterfly; the
+      // CTA partial of the row is published
       __syncthreads();
       ps[warp * 32 + lane] = Partial{amx, aidx, asum, anan};
       __syncthreads();
-      if (warp == 0 && lane < mt) {
-        Partial acc = ps[lane];
-        for (int w2 = 0; w2 < kWarps; ++w2)
-          for (int c2 = 0; c2 < kNCol; ++c2)
-            if (w2 != 0 || c2 != 0) partial_merge(acc, ps[w2 * 32 + c2 * kMTile + lane]);
-        g.part[(size_t)blockIdx.x * g.part_ld + m0 + lane] = acc;
+      for (int rr = warp; rr < mt; rr += kWarps) {
+        Partial acc{-INFINITY, 0x7fffffff, 0.f, 0};
+        for (int e = lane; e < kWarps * kNCol; e += 32)
+          partial_merge(acc, ps[(e / kNCol) * 32 + (e % kNCol) * kMTile + rr]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) partial_merge(acc, shfl_partial(acc, o));
+        if (lane == 0) g.part[(size_t)blockIdx.x * g.part_ld + m0 + rr] = acc;
       }
     }
   }
