@@ -36,8 +36,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
 # ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel sources whose
 # SHA-256 is recorded here; any other source reports traffic null.
-DRAM_BYTES_PER_PASS = 12.17e6
-DRAM_SOURCES_SHA256 = "c6f72a38673382cbc013233a9a6706918402159979d2fcb1e4fb47550b82db8e"
+DRAM_BYTES_PER_PASS = 12.09e6
+DRAM_SOURCES_SHA256 = "b2942b6c8a5be95f03d7412bf14766c4a347970df94a9ed8985173c140830fd2"
 
 
 def kernel_sources_sha256() -> str:
