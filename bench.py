@@ -30,6 +30,7 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 WORKLOAD = synth.MARIAN_GS
+STOP_RULE = "paper"          # "paper": StopC of Eq. 5; "prefix": accepted-prefix rule
 METRIC = "translated tokens/s at batch 1, GS-Jacobi vs greedy AR; HBM GB/s % of peak"
 FALLBACK_HBM_GBS = 6800.0
 
@@ -164,7 +165,7 @@ def oracle_tokens_per_s(weights, sentences, budget_s):
     tokens, t0, used = 0, time.perf_counter(), []
     for k, src in enumerate(sentences):
         step = od.model_step(model, src)
-        r = od.gs_jacobi(step, WORKLOAD.max_len(len(src)), WORKLOAD.b)
+        r = od.gs_jacobi(step, WORKLOAD.max_len(len(src)), WORKLOAD.b, stop_rule=STOP_RULE)
         tokens += len(r.tokens)
         used.append(k)
         if time.perf_counter() - t0 > budget_s:
@@ -194,7 +195,8 @@ def run_reference(args):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD.name, "sample": "one sentence per step, the "
+            "config": {"workload": WORKLOAD.name, "stop_rule": STOP_RULE,
+                       "sample": "one sentence per step, the "
                        "shortest sentences of the 256 (CPU oracle is slow)"},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                              "sample": f"{args.steps} sentences, GS-Jacobi b=5, numpy float64, "
@@ -241,7 +243,7 @@ def run_gpu(args):
     d_y = torch.zeros((n_s, max_tgt), dtype=torch.int32, device="cuda")
     d_info = torch.zeros((n_s, 4), dtype=torch.int32, device="cuda")
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
-    params = {m: [pkg.Decoder.params(m, WORKLOAD.max_len(len(s)), b=b)
+    params = {m: [pkg.Decoder.params(m, WORKLOAD.max_len(len(s)), b=b, stop_rule=STOP_RULE)
                   for s in sents]
               for m, b in (("gs_jacobi", WORKLOAD.b), ("greedy", 1), ("jacobi", 1),
                            ("hybrid_gs_jacobi", 3))}
@@ -309,7 +311,8 @@ def run_gpu(args):
     toks = []
     for k, s in enumerate(sents):
         dec.encode(s)
-        r = dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b, trace=True)
+        r = dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b, trace=True,
+                       stop_rule=STOP_RULE)
         assert r.n_iters == int(info[k, 1])
         total_bytes += decode_bytes(spec, len(s), r.trace)
         passes += r.n_iters
@@ -327,13 +330,14 @@ def run_gpu(args):
     for _ in range(args.warmup):
         for k, s in enumerate(sents[:8]):
             dec.encode(s)
-            dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b)
+            dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b, stop_rule=STOP_RULE)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(args.steps):
         for k, s in enumerate(sents):
             dec.encode(s)
-            r = dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b)
+            r = dec.decode("gs_jacobi", WORKLOAD.max_len(len(s)), b=WORKLOAD.b,
+                           stop_rule=STOP_RULE)
             e2e_tok += len(r.tokens)
             h2d += 4 * len(s)
             d2h += 4 + 16 + 4 * len(r.tokens)      # encode status, decode info, tokens
@@ -358,6 +362,7 @@ def run_gpu(args):
             "data": "synthetic: seeded N(0,0.02) weights, uniform random source ids",
             "config": {"workload": WORKLOAD.name if n_s == WORKLOAD.n_sentences else
                        f"{WORKLOAD.name} (first {n_s} sentences only)", "sentences_per_step": n_s,
+                       "stop_rule": STOP_RULE,
                        "timing": "CUDA events on the library stream; L2 flushed (256 MB write) "
                                  "between steps; replicas across GPUs"},
             "greedy": {"value": greedy_tps, "unit": "tokens/s",
@@ -402,10 +407,15 @@ def main():
                     help="GS-Jacobi block size (default: the workload's, 5)")
     ap.add_argument("--all-methods", action="store_true",
                     help="also time full-sentence Jacobi and Hybrid GS-Jacobi (b=3), one step each")
+    ap.add_argument("--stop-rule", default="paper", choices=["paper", "prefix"],
+                    help="when a block's passes end: paper = StopC of Eq. 5 (the block unchanged, "
+                         "or one pass per position); prefix = also once the unchanged leading "
+                         "tokens make the whole block exact")
     ap.add_argument("--sentences", type=int, default=0,
                     help="use only the first N sentences of the workload (profiling runs)")
     args = ap.parse_args()
-    global WORKLOAD
+    global WORKLOAD, STOP_RULE
+    STOP_RULE = args.stop_rule
     if args.workload == "marian-knob":
         WORKLOAD = synth.MARIAN_KNOB
     elif args.workload == "mbart":

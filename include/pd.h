@@ -104,6 +104,17 @@ pd_status pd_encode(pd_ctx* ctx, const int32_t* src, int n_src);
  * stream (ids are not range-checked; out-of-range ids are clamped on the device). */
 pd_status pd_encode_device(pd_ctx* ctx, const int32_t* d_src, int n_src);
 
+/* When a block's repeated passes end.  Both rules return the same tokens (after k passes the
+ * first k block positions are exact, Section 3.4, Proposition 1); they differ in passes.
+ *  PD_STOP_UNCHANGED: StopC of Eq. 5 (Section 3.3): the block ends when a pass leaves all of
+ *    its tokens unchanged, or after as many passes as the block has positions.
+ *  PD_STOP_PREFIX: also ends the block once the leading unchanged count c of a pass reaches
+ *    blk - 1: the first c + 1 new tokens are then exact (each was predicted from inputs
+ *    already equal to the solution), so the whole block is, and the confirming pass that
+ *    Eq. 5 needs is skipped.  The paper leaves other stopping conditions to future work
+ *    (Section 5, Conclusions); this is one, with the same result and at most as many passes. */
+typedef enum { PD_STOP_UNCHANGED = 0, PD_STOP_PREFIX = 1 } pd_stop_rule;
+
 typedef struct {
   int method;       /* pd_method */
   int b;            /* block size for GS-Jacobi / hybrid (>= 1); ignored by greedy, jacobi */
@@ -112,12 +123,13 @@ typedef struct {
   int h;            /* hybrid: parallel part up to position h (0 = max_len) */
   int stop_at_eos;  /* greedy / jacobi / gs_jacobi: end the returned y at the first EOS */
   int max_passes;   /* 0 = no limit; else stop with PD_ENOTCONV after this many passes */
+  int stop_rule;    /* pd_stop_rule (0 = Eq. 5) */
 } pd_decode_params;
 
 /* One decoder pass of the trace (DDGviz-style, Section 3.5): pass number (1-based), block
  * start position i (1-based), block length, number of leading block positions whose new
- * token equals the previous draft, StopC (Eq. 5) flag, index of the first EOS in the new
- * block tokens (-1 if none). */
+ * token equals the previous draft, StopC (Eq. 5) flag (under either stop rule), index of the
+ * first EOS in the new block tokens (-1 if none). */
 typedef struct {
   int32_t step, block_start, block_len, n_converged, stop, eos_idx;
 } pd_trace_step;

@@ -22,6 +22,7 @@ STATUS_NAMES = {0: "PD_OK", -1: "PD_EINVAL", -2: "PD_ENOMEM", -3: "PD_ECUDA", -4
                 -5: "PD_ENAN", -6: "PD_ESTATE", -7: "PD_ETIMEOUT"}
 
 METHODS = {"greedy": 0, "jacobi": 1, "gs_jacobi": 2, "hybrid_gs_jacobi": 3}
+STOP_RULES = {"paper": 0, "prefix": 1}      # pd_stop_rule: Eq. 5 StopC, accepted prefix
 
 # Every symbol include/pd.h declares.
 EXPORTED = ("pd_weights_nbytes", "pd_create", "pd_export_weights", "pd_encode",
@@ -47,7 +48,7 @@ class _Config(ctypes.Structure):
 
 class _DecodeParams(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("method", "b", "max_len", "h", "stop_at_eos",
-                                            "max_passes")]
+                                            "max_passes", "stop_rule")]
 
 
 class _TraceStep(ctypes.Structure):
@@ -192,14 +193,14 @@ class Decoder:
 
     @staticmethod
     def params(method: str, max_len: int, b: int = 1, h: int = 0, stop_at_eos: bool = True,
-               max_passes: int = 0) -> _DecodeParams:
+               max_passes: int = 0, stop_rule: str = "paper") -> _DecodeParams:
         return _DecodeParams(METHODS[method], int(b), int(max_len), int(h), int(stop_at_eos),
-                             int(max_passes))
+                             int(max_passes), STOP_RULES[stop_rule])
 
     def decode(self, method: str, max_len: int, b: int = 1, h: int = 0,
                stop_at_eos: bool = True, max_passes: int = 0,
-               trace: bool = False) -> DecodeResult:
-        p = self.params(method, max_len, b, h, stop_at_eos, max_passes)
+               trace: bool = False, stop_rule: str = "paper") -> DecodeResult:
+        p = self.params(method, max_len, b, h, stop_at_eos, max_passes, stop_rule)
         y = np.zeros(max_len, dtype=np.int32)
         n_y, n_it, n_tr = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
         if trace:

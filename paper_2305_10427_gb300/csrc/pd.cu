@@ -32,7 +32,7 @@ struct KParams {
   const int* enc_tok;       // encoder input ids (device)
   int debug_len;            // > 0: one teacher-forced pass over dbg_tok, logits out
   float* logits;            // [debug_len][V]
-  DecState init;            // method, b, max_len, h, stop_at_eos, max_passes
+  DecState init;            // method, b, max_len, h, stop_at_eos, max_passes, stop_rule
   int32_t* out_y;           // [max_len]
   int32_t* out_info;        // {n_y, n_iters, status, n_trace}
 };
@@ -394,7 +394,9 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
     if (s_nan) {
       ss.status = PD_ENAN; ss.n_y = i - 1; ss.done = 1;
     } else {
-      if (stop || ss.k >= blk) {                   // the block is solved
+      // the block is solved: StopC, the pass cap, or (accepted-prefix rule) the first c + 1
+      // new tokens exact with c + 1 >= blk
+      if (stop || ss.k >= blk || (ss.stop_rule == PD_STOP_PREFIX && c + 1 >= blk)) {
         const bool one_pos = ss.method == PD_GREEDY || ss.ar_tail;
         if (one_pos) {
           const bool eos_ends = ss.ar_tail ? true : (ss.stop_at_eos != 0);
@@ -873,6 +875,7 @@ pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int32_t* d_y, int32_
   P.init.h = (p->h <= 0 || p->h > p->max_len) ? p->max_len : p->h;
   P.init.stop_at_eos = p->stop_at_eos;
   P.init.max_passes = p->max_passes;
+  P.init.stop_rule = p->stop_rule;
   P.out_y = d_y;
   P.out_info = d_info;
   return launch<W>(c, false, P);
@@ -894,6 +897,8 @@ pd_status check_params(pd_ctx* c, const pd_decode_params* p) {
   if ((p->method == PD_GS_JACOBI || p->method == PD_HYBRID_GS_JACOBI) && p->b < 1)
     return fail(c, PD_EINVAL, "b must be >= 1");
   if (p->max_passes < 0) return fail(c, PD_EINVAL, "max_passes must be >= 0");
+  if (p->stop_rule != PD_STOP_UNCHANGED && p->stop_rule != PD_STOP_PREFIX)
+    return fail(c, PD_EINVAL, "stop_rule");
   if (c->cfg.learned_pos && p->max_len > c->cfg.max_pos)
     return fail(c, PD_EINVAL, "max_len exceeds the learned position table");
   if (!c->encoded) return fail(c, PD_ESTATE, "pd_decode before pd_encode");

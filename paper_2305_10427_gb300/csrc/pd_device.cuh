@@ -74,7 +74,7 @@ struct Partial {
 
 // Decoding state, in device memory, advanced by the commit step.
 struct DecState {
-  int method, b, max_len, h, stop_at_eos, max_passes;
+  int method, b, max_len, h, stop_at_eos, max_passes, stop_rule;
   int b_eff, m_eff;       // current block size rule and system size (h for hybrid)
   int i, blk, k;          // block start (1-based), block length, passes in this block
   int ar_tail;            // hybrid: past h, one position per pass

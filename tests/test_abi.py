@@ -77,3 +77,44 @@ def test_null_context_calls(lib):
     assert lib.pd_launch_count(None) == 0
     assert lib.pd_last_error(None) == b"context is NULL"
     lib.pd_destroy(None)
+
+
+def _header_text():
+    return re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+
+
+def _struct_fields(text, name):
+    body = re.search(r"typedef struct \{([^{}]*)\}\s*" + name + r"\s*;", text).group(1)
+    out = []
+    for decl in body.split(";"):
+        decl = decl.strip()
+        if decl:
+            out += [n.strip() for n in decl.split(None, 1)[1].split(",")]
+    return out
+
+
+def _enum_values(text, name):
+    body = re.search(r"typedef enum \{([^{}]*)\}\s*" + name + r"\s*;", text).group(1)
+    return {k: int(v) for k, v in re.findall(r"(PD_[A-Z0-9_]+)\s*=\s*(-?\d+)", body)}
+
+
+@pytest.mark.parametrize("cname,cls", [("pd_config", B._Config),
+                                       ("pd_decode_params", B._DecodeParams),
+                                       ("pd_trace_step", B._TraceStep)])
+def test_binding_structs_match_header(cname, cls):
+    """The ctypes mirrors declare the header's fields in the header's order (every field is a
+    4-byte int or float, so equal order means equal layout)."""
+    assert _struct_fields(_header_text(), cname) == [f for f, _ in cls._fields_]
+    assert ctypes.sizeof(cls) == 4 * len(cls._fields_)
+
+
+def test_binding_enums_match_header():
+    text = _header_text()
+    assert _enum_values(text, "pd_method") == {
+        "PD_GREEDY": B.METHODS["greedy"], "PD_JACOBI": B.METHODS["jacobi"],
+        "PD_GS_JACOBI": B.METHODS["gs_jacobi"],
+        "PD_HYBRID_GS_JACOBI": B.METHODS["hybrid_gs_jacobi"]}
+    assert _enum_values(text, "pd_stop_rule") == {"PD_STOP_UNCHANGED": B.STOP_RULES["paper"],
+                                                  "PD_STOP_PREFIX": B.STOP_RULES["prefix"]}
+    status = _enum_values(text, "pd_status")
+    assert {v: k for k, v in status.items()} == B.STATUS_NAMES

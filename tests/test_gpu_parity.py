@@ -13,6 +13,8 @@ Checks, per the method's guarantees:
 * edge cases (one-token source, max_len 1, b > max_len, b = 1, EOS-heavy model) and error
   statuses (bad arguments, decode before encode, pass budget, NaN weights).
 """
+import ctypes
+
 import numpy as np
 import pytest
 
@@ -103,6 +105,16 @@ def tiny_eos():
 
 
 @pytest.fixture(scope="module")
+def tiny_fast():
+    """Tiny model whose predictions hardly depend on the input tokens (token-embedding scale
+    0.002): blocks converge early, and on the 16-id sentence GS-Jacobi b=5 takes 11 passes under
+    Eq. 5 and 10 under the accepted-prefix rule, every oracle decision with margin > 1e-3."""
+    s = Setup(synth.TINY, 64, 64, seed=6, embed_std=0.002)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
 def marian():
     s = Setup(synth.MARIAN, 64, 128, seed=0)
     yield s
@@ -134,6 +146,18 @@ def all_methods(dec, max_len, stop_at_eos=True):
     return out
 
 
+def assert_same_run(got, ref, name):
+    """GPU run == oracle run: tokens, pass count, and every trace row with its tokens."""
+    assert got.tokens == ref.tokens, name
+    assert got.n_iters == ref.n_iters, name
+    assert len(got.trace) == len(ref.trace), name
+    for t, (a, r) in enumerate(zip(got.trace, ref.trace)):
+        assert (a["step"], a["block_start"], a["block_len"], a["n_converged"], bool(a["stop"]),
+                a["eos_idx"]) == (r.step, r.block_start, r.block_len, r.n_converged, r.stop,
+                                  r.eos_idx), (name, t)
+        assert list(got.trace_tokens[t][:a["block_len"]]) == r.tokens, (name, t)
+
+
 def compare_with_oracle_runs(setup, src, max_len, res):
     """Pass counts and traces equal the oracle's run where all its decisions had margin."""
     step = setup.step(src)
@@ -148,17 +172,26 @@ def compare_with_oracle_runs(setup, src, max_len, res):
         ref = run()
         if ref.min_margin <= setup.margin:
             continue
-        got = res[name]
-        assert got.tokens == ref.tokens, name
-        assert got.n_iters == ref.n_iters, name
-        assert len(got.trace) == len(ref.trace), name
-        for t, (a, r) in enumerate(zip(got.trace, ref.trace)):
-            assert (a["step"], a["block_start"], a["block_len"], a["n_converged"], bool(a["stop"]),
-                    a["eos_idx"]) == (r.step, r.block_start, r.block_len, r.n_converged, r.stop,
-                                      r.eos_idx), (name, t)
-            assert list(got.trace_tokens[t][:a["block_len"]]) == r.tokens, (name, t)
+        assert_same_run(res[name], ref, name)
         compared += 1
     return compared
+
+
+def block_ends_follow_rule(trace, rule):
+    """Every block of a GPU trace ends at its first pass where the rule holds: StopC (Eq. 5),
+    the pass cap (k == blk), or, for the accepted-prefix rule, c + 1 >= blk."""
+    k = 0
+    for t, row in enumerate(trace):
+        k += 1
+        c, blk = row["n_converged"], row["block_len"]
+        ends = bool(row["stop"]) or k == blk or (rule == "prefix" and c + 1 >= blk)
+        last_of_block = t + 1 == len(trace) or trace[t + 1]["block_start"] != row["block_start"]
+        if not last_of_block:
+            assert not ends, (t, row)
+        else:
+            k = 0
+            if t + 1 < len(trace):
+                assert ends, (t, row)
 
 
 # ---- weights -------------------------------------------------------------------------------
@@ -212,6 +245,48 @@ def test_tiny_all_methods(name, request):
         check_tokens_teacher_forced(s, src, g)
         compared += compare_with_oracle_runs(s, src, max_len, res)
     assert compared >= 8
+
+
+PREFIX_RUNS = (("jacobi", 0), ("gs_jacobi", 3), ("gs_jacobi", 5), ("hybrid_gs_jacobi", 3))
+
+
+def oracle_run(step, method, max_len, b, eos, rule):
+    if method == "jacobi":
+        return od.jacobi(step, max_len, eos=eos, stop_rule=rule)
+    if method == "gs_jacobi":
+        return od.gs_jacobi(step, max_len, b, eos=eos, stop_rule=rule)
+    return od.hybrid_gs_jacobi(step, max_len, b, eos=eos, stop_rule=rule)
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny_vary", "tiny_eos", "tiny_fast"])
+def test_prefix_stop_rule(name, request):
+    """Accepted-prefix stop rule: the greedy tokens, never more passes than Eq. 5's rule (the
+    passes of a block are the same until the prefix rule ends it), block ends where the rule
+    says, and the oracle's run (pass counts, traces) wherever its decisions had margin."""
+    s = request.getfixturevalue(name)
+    srcs = [synth.TINY_JACOBI.sentences()[0]] + synth.sentences(21, 3, 5, 30, s.spec.vocab)
+    saved = compared = 0
+    for src in srcs:
+        max_len = 16 if len(src) == 16 else 2 * len(src)
+        s.dec.encode(src)
+        g = s.dec.decode("greedy", max_len)
+        step = s.step(src)
+        for m, b in PREFIX_RUNS:
+            pre = s.dec.decode(m, max_len, b=b, trace=True, stop_rule="prefix")
+            pap = s.dec.decode(m, max_len, b=b, trace=True)
+            assert pre.tokens == g.tokens, (m, b)
+            assert pre.n_iters <= pap.n_iters, (m, b)
+            saved += pap.n_iters - pre.n_iters
+            block_ends_follow_rule(pre.trace, "prefix")
+            block_ends_follow_rule(pap.trace, "paper")
+            ref = oracle_run(step, m, max_len, b, s.eos, "prefix")
+            if ref.min_margin > s.margin:
+                assert_same_run(pre, ref, (m, b))
+                compared += 1
+    if name in ("tiny_vary", "tiny_eos", "tiny_fast"):
+        assert saved > 0
+    if name in ("tiny", "tiny_fast"):
+        assert compared >= 1
 
 
 def test_tiny_eos_paths(tiny_eos):
@@ -322,6 +397,14 @@ def test_errors(tiny):
         with pytest.raises(pkg.PdError) as e:
             fresh.decode("gs_jacobi", **kw)
         assert e.value.status == -1
+    p = fresh.params("gs_jacobi", 4, b=2)
+    p.stop_rule = 7                                                 # no such pd_stop_rule
+    y = np.zeros(4, dtype=np.int32)
+    n_y, n_it = ctypes.c_int(), ctypes.c_int()
+    st = fresh._lib.pd_decode(fresh._h, ctypes.byref(p),
+                              y.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
+                              ctypes.byref(n_y), ctypes.byref(n_it), None, None, None, 0, None)
+    assert st == -1
     fresh.close()
 
 
