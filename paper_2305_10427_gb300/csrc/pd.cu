@@ -226,7 +226,7 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const in
       g.slot0 = pos0;
       break;
     case PH_O:                          // self-attention output + residual
-      g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
+      g.N = D.d; g.K = D.d; g.xw_src = B.att; g.w = L.wo; g.bias = L.bo;
       g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = (pre || l == 0) ? B.ra : B.xa;
       break;
     case PH_QC:                         // cross-attention query
@@ -236,17 +236,17 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const in
       g.w = L.wqc; g.bias = L.bqc; g.epi = EPI_STORE; g.out = B.q; g.ld = D.d;
       break;
     case PH_OC:                         // cross-attention output + residual
-      g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.woc; g.bias = L.boc;
+      g.N = D.d; g.K = D.d; g.xw_src = B.att; g.w = L.woc; g.bias = L.boc;
       g.epi = EPI_RESID; g.out = B.rc; g.ld = D.d; g.resid = pre ? B.rb : B.xb;
       break;
     case PH_FFN1:
       g.N = D.f; g.K = D.d; g.x_src = B.rc;
       if (pre) { g.ln_b_g = L.ln3g; g.ln_b_b = L.ln3b; }
       else { g.ln_a_g = L.ln2g; g.ln_a_b = L.ln2b; g.x_store = B.xc; }
-      g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
+      g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out_w = B.ffh; g.ld = D.f;
       break;
     case PH_FFN2:
-      g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
+      g.N = D.d; g.K = D.f; g.xw_src = B.ffh; g.w = L.w2; g.bias = L.b2;
       g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = pre ? B.rc : B.xc;
       break;
   }
@@ -304,10 +304,10 @@ __device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, f
     if (attn) {
       const int l = ph >> 3;
       if ((ph & 7) == PH_SELF)
-        attn_phase<W>(D, B.q, B.kself + (size_t)l * D.max_tgt * D.d,
+        attn_phase<W, W>(D, B.q, B.kself + (size_t)l * D.max_tgt * D.d,
                       B.vself + (size_t)l * D.max_tgt * D.d, B.att, M, pos0, 0, scratch);
       else
-        attn_phase<W>(D, B.q, B.kcross + (size_t)l * D.max_src * D.d,
+        attn_phase<W, W>(D, B.q, B.kcross + (size_t)l * D.max_src * D.d,
                       B.vcross + (size_t)l * D.max_src * D.d, B.att, M, -1, P.n_src, scratch);
     } else {
       gemm_phase<W>(ga, T, D, smem);
@@ -574,11 +574,11 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
-    attn_phase<float>(D, B.q, B.k, B.v, B.att, n, -1, n, scratch);
+    attn_phase<float, W>(D, B.q, B.k, B.v, B.att, n, -1, n, scratch);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
     g = GemmArgs<W>{};
-    g.M = n; g.N = D.d; g.K = D.d; g.x_src = B.att; g.w = L.wo; g.bias = L.bo;
+    g.M = n; g.N = D.d; g.K = D.d; g.xw_src = B.att; g.w = L.wo; g.bias = L.bo;
     g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
     gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
@@ -589,13 +589,13 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     if (pre) { g.ln_b_g = L.ln2g; g.ln_b_b = L.ln2b; }
     else { g.ln_a_g = L.ln1g; g.ln_a_b = L.ln1b; g.x_store = B.xb; }
     const float* res2 = pre ? B.rb : B.xb;
-    g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out = B.ffh; g.ld = D.f;
+    g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out_w = B.ffh; g.ld = D.f;
     gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
     g = GemmArgs<W>{};
-    g.M = n; g.N = D.d; g.K = D.f; g.x_src = B.ffh; g.w = L.w2; g.bias = L.b2;
+    g.M = n; g.N = D.d; g.K = D.f; g.xw_src = B.ffh; g.w = L.w2; g.bias = L.b2;
     g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res2;
     gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);

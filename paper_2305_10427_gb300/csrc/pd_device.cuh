@@ -29,7 +29,7 @@ constexpr unsigned long long kWaitNs = 10000000000ull;  // bounded device waits:
 
 enum Epi : int {
   EPI_STORE = 0,     // out = acc + bias
-  EPI_ACT = 1,       // out = act(acc + bias)
+  EPI_ACT = 1,       // out_w = act(acc + bias), rounded to the weight type
   EPI_RESID = 2,     // out = acc + bias + resid
   EPI_QKV = 3,       // [q | k | v] = acc + bias -> q rows, k/v to cache slots
   EPI_KVCROSS = 4,   // columns of all decoder layers' [k | v] cross projections -> caches
@@ -85,8 +85,9 @@ template <typename W>
 struct Bufs {
   float *ra, *rb, *rc;         // residual-stream rows [rows][d]
   float *xa, *xb, *xc;         // normalised sublayer inputs (post-LN residuals) [rows][d]
-  float *q, *k, *v, *att;      // [rows][d]
-  float* ffh;                  // [rows][f]
+  float *q, *k, *v;            // [rows][d]
+  W* att;                      // [rows][d] attention output, rounded to W (the O input type)
+  W* ffh;                      // [rows][f] FFN hidden, rounded to W (FFN2's input type)
   W *kself, *vself;            // [Ld][max_tgt][d]
   W *kcross, *vcross;          // [Ld][max_src][d]
   Partial* part;               // [grid][rows]
@@ -331,6 +332,7 @@ struct GemmArgs {
   // E[tok] * sqrt(d) + position(pos0 + m); then optionally LayerNorm ln_a, the result stored
   // to x_store (fp32, by CTA 0), then optionally LayerNorm ln_b; X is rounded to W.
   const float* x_src;
+  const W* xw_src;          // input rows already rounded to W (plain copy; instead of x_src)
   const int* emb_tok;
   int emb_pos0;
   const W *ln_a_g, *ln_a_b;
@@ -339,7 +341,8 @@ struct GemmArgs {
   const W* w;               // [N][K]
   const W* bias;            // [N] or nullptr
   int epi;
-  float* out;               // [M][ld] for STORE / ACT / RESID / LOGITS; q rows for QKV
+  float* out;               // [M][ld] for STORE / RESID / LOGITS; q rows for QKV
+  W* out_w;                 // [M][ld] for ACT
   int ld;
   const float* resid;       // [M][ld]
   W *kdst, *vdst;           // QKV: cache rows (slot = slot0 + m); KVCROSS: cross caches
@@ -462,10 +465,10 @@ __device__ __forceinline__ float dot_part(const float* __restrict__ w, int K, in
 
 constexpr int kMaxRowRegs = 8;      // embedded / normalised rows: <= 8 float4 per lane
 constexpr int kStageB = 4;
-__device__ __forceinline__ float4 ld_act4(const float* p) {
-  float4 v;
-  asm volatile("ld.global.cg.v4.f32 {%0,%1,%2,%3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+__device__ __forceinline__ uint4 ld_act16(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                : "l"(p));
   return v;
 }
@@ -525,26 +528,39 @@ __device__ void stage_x(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims&
   const int warp = threadIdx.x >> 5;
   const int K = g.K;
   const bool any_ln = g.ln_a_g != nullptr || g.ln_b_g != nullptr || g.emb_tok != nullptr;
-  if (!any_ln) {                         // plain copy (any K multiple of 128), all threads
+  if (!any_ln) {
+    // plain copy, all threads, 16-byte items: fp32 rows (4 elements, rounded to W, optionally
+    // stored to x_store) or rows already in W (16 / sizeof(W) elements, copied as they are)
+    const bool wsrc = g.xw_src != nullptr;
     const bool store = g.x_store != nullptr && blockIdx.x == 0;
-    const int K4 = K / 4, F = mt * K4;
+    const int E = wsrc ? 16 / (int)sizeof(W) : 4;
+    const int es = wsrc ? (int)sizeof(W) : 4;
+    const char* src = wsrc ? reinterpret_cast<const char*>(g.xw_src)
+                           : reinterpret_cast<const char*>(g.x_src);
+    const int KE = K / E, F = mt * KE;
     for (int f0 = 0; f0 < F; f0 += kThreads * kStageB) {
-      float4 v[kStageB];
+      uint4 v[kStageB];
 #pragma unroll
       for (int j = 0; j < kStageB; ++j) {
         const int f = f0 + j * kThreads + (int)threadIdx.x;
         if (f < F) {
-          const int r = f / K4, k = (f - r * K4) * 4;
-          v[j] = ld_act4(g.x_src + (size_t)(m0 + r) * K + k);
+          const int r = f / KE, k = (f - r * KE) * E;
+          v[j] = ld_act16(src + ((size_t)(m0 + r) * K + k) * es);
         }
       }
 #pragma unroll
       for (int j = 0; j < kStageB; ++j) {
         const int f = f0 + j * kThreads + (int)threadIdx.x;
         if (f < F) {
-          const int r = f / K4, k = (f - r * K4) * 4;
-          if (store) *reinterpret_cast<float4*>(g.x_store + (size_t)(m0 + r) * K + k) = v[j];
-          put4(xs + (size_t)r * K + k, v[j]);
+          const int r = f / KE, k = (f - r * KE) * E;
+          if (wsrc) {
+            *reinterpret_cast<uint4*>(xs + (size_t)r * K + k) = v[j];
+          } else {
+            const float4 x = make_float4(__uint_as_float(v[j].x), __uint_as_float(v[j].y),
+                                         __uint_as_float(v[j].z), __uint_as_float(v[j].w));
+            if (store) *reinterpret_cast<float4*>(g.x_store + (size_t)(m0 + r) * K + k) = x;
+            put4(xs + (size_t)r * K + k, x);
+          }
         }
       }
     }
@@ -711,7 +727,7 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
       const float v = a + bias;
       switch (g.epi) {
         case EPI_STORE: g.out[(size_t)m * g.ld + n] = v; break;
-        case EPI_ACT: g.out[(size_t)m * g.ld + n] = act_fn(v, D.act); break;
+        case EPI_ACT: g.out_w[(size_t)m * g.ld + n] = from_f<W>(act_fn(v, D.act)); break;
         case EPI_RESID: g.out[(size_t)m * g.ld + n] = v + g.resid[(size_t)m * g.ld + n]; break;
         case EPI_QKV: {
           const int which = n / D.d, cc = n - which * D.d;
@@ -758,7 +774,7 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
 }
 
 // ------------------------------------------------------------------------------------------
-// attention: out[m, head] = softmax(q k^T / sqrt(dh)) v over keys 0..T(m)-1
+// attention: out[m, head] = softmax(q k^T / sqrt(dh)) v over keys 0..T(m)-1, stored as O
 // ------------------------------------------------------------------------------------------
 
 template <typename KV>
@@ -815,9 +831,9 @@ __device__ __forceinline__ void add_pv32(const float* v, float p, float (&acc)[3
 // p-weighted value sums are accumulated per lane in ascending key order, then combined by
 // fixed butterflies, so a row's result depends only on its own query and keys.
 // causal_pos0 >= 0: row m attends keys 0..causal_pos0+m; else all n_keys keys.
-template <typename KV>
+template <typename KV, typename O>
 __device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV* kc, const KV* vc,
-                           float* out, int M, int causal_pos0, int n_keys, float* scratch) {
+                           O* out, int M, int causal_pos0, int n_keys, float* scratch) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int gw = warp * gridDim.x + blockIdx.x;     // items dealt to CTAs round robin
@@ -854,7 +870,7 @@ __device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV*
         add_pv32(vc + (size_t)j * D.d + h * dh + c0, p, acc);
       }
       const float tot = reduce_scatter32(acc);
-      out[(size_t)m * D.d + h * dh + c0 + lane] = tot / sum;
+      out[(size_t)m * D.d + h * dh + c0 + lane] = from_f<O>(tot / sum);
     }
     __syncwarp();
   }
