@@ -312,7 +312,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, f
     } else {
       gemm_phase<W>(ga, T, D, smem);
     }
-    if (ph == nph - 1) break;            // the LM head ends at the caller's commit barrier
+    if (ph == nph - 1) break;            // the caller's barrier follows the LM head
     const int next = is_attn_phase(ph + 1, nph) ? ph + 2 : ph + 1;
     if (!grid_barrier(B.bar, tgt, status, [&] {
           if (!attn && threadIdx.x == 32) gemm_args(P, next, M, pos0, tok, logits, ga);
@@ -324,12 +324,19 @@ __device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, f
 }
 
 // ------------------------------------------------------------------------------------------
-// fixed-point commit (one CTA): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
+// fixed-point commit (every CTA): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
 // ------------------------------------------------------------------------------------------
 
-// The decoding state is copied into shared memory with one load per field (issued together),
-// the block's previous draft likewise; one thread then takes the decisions from shared memory
-// and the results are written back in parallel.
+template <typename W>
+__device__ __forceinline__ DecState& smem_state() {
+  __shared__ DecState s;
+  return s;
+}
+
+// Run after the grid barrier that follows the LM head, by every CTA on its own copy of the
+// state and of y (shared memory): the CTA partials of each row are merged in the same fixed
+// order everywhere, so every CTA takes the same decisions and needs nothing from the others.
+// CTA 0 alone writes the trace to device memory.
 template <typename W>
 __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   const Dims& D = P.D;
@@ -337,22 +344,31 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   const SmemLayout SL = smem_layout(D, sizeof(W));
   int* ntok = reinterpret_cast<int*>(smem + SL.commit);
   float* nprob = reinterpret_cast<float*>(ntok + D.max_tgt + 1);
-  int* yold = reinterpret_cast<int*>(nprob + D.max_tgt + 1);
-  constexpr int kNS = (int)(sizeof(DecState) / sizeof(int));
-  __shared__ DecState ss;
-  __shared__ int s_nan, s_eos;
+  int* sy = reinterpret_cast<int*>(nprob + D.max_tgt + 1);       // y_0..y_m
+  DecState& ss = smem_state<W>();
+  __shared__ int s_nan, s_scan;
   const int tid = threadIdx.x;
   const int lane = tid & 31, warp = tid >> 5;
-  if (tid < kNS) reinterpret_cast<int*>(&ss)[tid] = __ldcg(reinterpret_cast<const int*>(B.st) + tid);
-  if (tid == 0) { s_nan = 0; s_eos = 0x7fffffff; }
+  const int blk = ss.blk, i = ss.i, t = ss.n_trace;   // read before thread 0 changes ss
+  if (tid == 0) { s_nan = 0; s_scan = 0; }
   __syncthreads();
-  const int blk = ss.blk, i = ss.i;
-  for (int r = tid; r < blk; r += blockDim.x) yold[r] = __ldcg(B.y + i + r);
-  // per row: the CTA partials merged lane-wise in ascending CTA order, then by a fixed
-  // butterfly (the merge is symmetric, so every lane ends with the same result)
+  // per row: the CTA partials merged lane-wise in ascending CTA order (loads issued in
+  // batches), then by a fixed butterfly (the merge is symmetric, so every lane ends with the
+  // same result)
+  constexpr int kBatch = 8;
   for (int r = warp; r < blk; r += kWarps) {
     Partial a{-INFINITY, 0x7fffffff, 0.f, 0};
-    for (int c = lane; c < (int)gridDim.x; c += 32) partial_merge(a, B.part[(size_t)c * D.rows + r]);
+    for (int c0 = 0; c0 < (int)gridDim.x; c0 += 32 * kBatch) {
+      Partial v[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int c = c0 + 32 * j + lane;
+        if (c < (int)gridDim.x) v[j] = B.part[(size_t)c * D.rows + r];
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j)
+        if (c0 + 32 * j + lane < (int)gridDim.x) partial_merge(a, v[j]);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const Partial b = shfl_partial(a, o);
@@ -365,18 +381,15 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
     }
   }
   __syncthreads();
-  const int t = ss.n_trace;
-  for (int r = tid; r < blk; r += blockDim.x) {
-    B.y[i + r] = ntok[r];
-    if (t < D.max_tgt) {
+  if (blockIdx.x == 0 && t < D.max_tgt) {
+    for (int r = tid; r < blk; r += blockDim.x) {
       B.trace_tok[(size_t)t * D.max_tgt + r] = ntok[r];
       B.trace_prob[(size_t)t * D.max_tgt + r] = nprob[r];
     }
   }
-  bool scan = false;                                // search y_1..y_m for the first EOS
   if (tid == 0) {
-    int c = 0;
-    while (c < blk && ntok[c] == yold[c]) ++c;
+    int c = 0;                                     // leading positions equal to the old draft
+    while (c < blk && ntok[c] == sy[i + c]) ++c;
     const int stop = c == blk;
     int eos_idx = -1;
     for (int r = 0; r < blk; ++r)
@@ -385,10 +398,12 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
     const int n_it = ss.n_iters + 1;
     ss.n_iters = n_it;
     if (t < D.max_tgt) {
-      pd_trace_step row;
-      row.step = n_it; row.block_start = i; row.block_len = blk; row.n_converged = c;
-      row.stop = stop; row.eos_idx = eos_idx;
-      B.trace[t] = row;
+      if (blockIdx.x == 0) {
+        pd_trace_step row;
+        row.step = n_it; row.block_start = i; row.block_len = blk; row.n_converged = c;
+        row.stop = stop; row.eos_idx = eos_idx;
+        B.trace[t] = row;
+      }
       ss.n_trace = t + 1;
     }
     if (s_nan) {
@@ -415,7 +430,7 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
           if (ni > ss.m_eff) {
             ss.done = 1;
             ss.n_y = ss.m_eff;
-            scan = (ss.method == PD_JACOBI || ss.method == PD_GS_JACOBI) && ss.stop_at_eos;
+            s_scan = (ss.method == PD_JACOBI || ss.method == PD_GS_JACOBI) && ss.stop_at_eos;
           } else {
             ss.i = ni;
             const int rest = ss.m_eff - ni + 1;
@@ -432,36 +447,36 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
         ss.done = 1;
       }
     }
-    if (scan) s_eos = -1;                          // ask for the scan below
   }
   __syncthreads();
-  if (s_eos == -1) {                               // first EOS among y_1..y_m (written above)
-    __syncthreads();
-    if (tid == 0) s_eos = 0x7fffffff;
-    __syncthreads();
-    for (int p = 1 + tid; p <= ss.m_eff; p += blockDim.x)
-      if (__ldcg(B.y + p) == D.eos) atomicMin(&s_eos, p);
-    __syncthreads();
-    if (tid == 0 && s_eos != 0x7fffffff) ss.n_y = s_eos;
-    __syncthreads();
+  for (int r = tid; r < blk; r += blockDim.x) sy[i + r] = ntok[r];   // y_{i:i+blk} <- new
+  __syncthreads();
+  if (s_scan && tid == 0) {                        // the first EOS among y_1..y_m ends y
+    for (int p = 1; p <= ss.m_eff; ++p)
+      if (sy[p] == D.eos) { ss.n_y = p; break; }
   }
-  // write the state back; a non-zero status is only ever set, never cleared
-  if (tid < kNS && tid != (int)(offsetof(DecState, status) / sizeof(int)))
-    reinterpret_cast<int*>(B.st)[tid] = reinterpret_cast<const int*>(&ss)[tid];
-  if (tid == 0 && ss.status != 0) atomicCAS(&B.st->status, 0, ss.status);
+  __syncthreads();
 }
 
+// CTA 0, at the end of a decode: tokens and info from its copy of the state; a failure a
+// device-side wait recorded in the status word (PD_ETIMEOUT) takes precedence.
 template <typename W>
-__device__ void write_outputs(const KParams<W>& P) {
-  volatile DecState* s = P.B.st;
+__device__ void write_outputs(const KParams<W>& P, const unsigned char* smem) {
+  const Dims& D = P.D;
+  const SmemLayout SL = smem_layout(D, sizeof(W));
+  const int* sy = reinterpret_cast<const int*>(smem + SL.commit) + 2 * (D.max_tgt + 1);
+  const DecState& ss = smem_state<W>();
+  __syncthreads();
+  if (threadIdx.x == 0 && ss.status != 0) atomicCAS(&P.B.st->status, 0, ss.status);
   if (P.out_info == nullptr) return;
-  const int n_y = s->n_y;
-  for (int p = threadIdx.x; p < n_y; p += blockDim.x) P.out_y[p] = P.B.y[1 + p];
+  const int n_y = ss.n_y;
+  for (int p = threadIdx.x; p < n_y; p += blockDim.x) P.out_y[p] = sy[1 + p];
   if (threadIdx.x == 0) {
+    const int g = atomicAdd(&P.B.st->status, 0);
     P.out_info[0] = n_y;
-    P.out_info[1] = s->n_iters;
-    P.out_info[2] = s->status;
-    P.out_info[3] = s->n_trace;
+    P.out_info[1] = ss.n_iters;
+    P.out_info[2] = g;
+    P.out_info[3] = ss.n_trace;
   }
 }
 
@@ -472,7 +487,6 @@ __device__ void write_outputs(const KParams<W>& P) {
 template <typename W>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   extern __shared__ __align__(16) unsigned char smem[];
-  __shared__ int s_done, s_i, s_blk;
   unsigned tgt = 0;
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
@@ -490,45 +504,37 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
     return;
   }
 
-  if (blockIdx.x == 0) {
-    for (int p = threadIdx.x; p <= P.init.max_len; p += blockDim.x)
-      B.y[p] = p == 0 ? D.bos : D.pad;                       // InitT: all PAD (Section 3.3)
-    if (threadIdx.x == 0) {
-      DecState s = P.init;
-      s.b_eff = s.method == PD_GREEDY ? 1 : (s.method == PD_JACOBI ? s.max_len : s.b);
-      s.m_eff = s.method == PD_HYBRID_GS_JACOBI ? s.h : s.max_len;
-      s.i = 1;
-      s.blk = s.b_eff < s.m_eff ? s.b_eff : s.m_eff;
-      s.k = 0; s.ar_tail = 0; s.n_iters = 0; s.done = 0; s.n_y = 0; s.n_trace = 0;
-      s.status = 0;
-      *B.st = s;
-    }
+  // every CTA: its copy of the state and of y_0..y_m; InitT = all PAD (Section 3.3)
+  const SmemLayout SL = smem_layout(D, sizeof(W));
+  int* sy = reinterpret_cast<int*>(smem + SL.commit) + 2 * (D.max_tgt + 1);
+  DecState& ss = smem_state<W>();
+  for (int p = threadIdx.x; p <= P.init.max_len; p += blockDim.x) sy[p] = p == 0 ? D.bos : D.pad;
+  if (threadIdx.x == 0) {
+    DecState s = P.init;
+    s.b_eff = s.method == PD_GREEDY ? 1 : (s.method == PD_JACOBI ? s.max_len : s.b);
+    s.m_eff = s.method == PD_HYBRID_GS_JACOBI ? s.h : s.max_len;
+    s.i = 1;
+    s.blk = s.b_eff < s.m_eff ? s.b_eff : s.m_eff;
+    s.k = 0; s.ar_tail = 0; s.n_iters = 0; s.done = 0; s.n_y = 0; s.n_trace = 0;
+    s.status = 0;
+    ss = s;
+    if (blockIdx.x == 0) *status = 0;       // nothing reads it before the first barrier wait
   }
-  if (!grid_barrier(B.bar, tgt, status)) { if (blockIdx.x == 0) write_outputs(P); return; }
+  __syncthreads();
 
   for (;;) {
-    if (threadIdx.x == 0) {
-      volatile DecState* s = B.st;
-      s_done = s->done;
-      s_i = s->i;
-      s_blk = s->blk;
-    }
-    __syncthreads();
-    if (s_done) break;
-    const int M = s_blk, pos0 = s_i - 1;
+    if (ss.done) break;
+    const int M = ss.blk, pos0 = ss.i - 1;
     // row r's input is the token at position i-1+r: y_{i-1}, then the block's draft
     // (the shift-left of Algorithm 2's appendix note)
-    if (!run_pass<W>(P, M, pos0, B.y + pos0, nullptr, tgt, smem)) break;
-    // the last CTA to finish its LM-head columns merges the argmax partials and commits
-    if (!grid_barrier_last(B.bar, tgt, status, [&] { commit<W>(P, smem); })) break;
+    if (!run_pass<W>(P, M, pos0, sy + pos0, nullptr, tgt, smem)) break;
+    if (!grid_barrier(B.bar, tgt, status)) break;
+    commit<W>(P, smem);
   }
 #ifdef PD_TIMELINE
   tl_dump();
 #endif
-  if (blockIdx.x == 0) {
-    __syncthreads();
-    write_outputs(P);
-  }
+  if (blockIdx.x == 0) write_outputs(P, smem);
 }
 
 template <typename W>
@@ -799,7 +805,6 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
   PD_TRY(dalloc(c, &B.kcross, (size_t)D.Ld * D.max_src * d));
   PD_TRY(dalloc(c, &B.vcross, (size_t)D.Ld * D.max_src * d));
   PD_TRY(dalloc(c, &B.part, (size_t)c->grid * R));
-  PD_TRY(dalloc(c, &B.y, (size_t)D.max_tgt + 1));
   PD_TRY(dalloc(c, &B.st, 1));
   PD_TRY(dalloc(c, &B.trace, (size_t)D.max_tgt));
   PD_TRY(dalloc(c, &B.trace_tok, (size_t)D.max_tgt * D.max_tgt));

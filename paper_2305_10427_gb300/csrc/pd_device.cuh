@@ -72,7 +72,9 @@ struct Partial {
   int nan;       // a NaN logit was seen
 };
 
-// Decoding state, in device memory, advanced by the commit step.
+// Decoding state.  Every CTA keeps its own copy in shared memory and advances it by the same
+// commit step from the same merged LM-head partials, so the copies stay identical; CTA 0
+// writes the final one to device memory.
 struct DecState {
   int method, b, max_len, h, stop_at_eos, max_passes, stop_rule;
   int b_eff, m_eff;       // current block size rule and system size (h for hybrid)
@@ -91,7 +93,6 @@ struct Bufs {
   W *kself, *vself;            // [Ld][max_tgt][d]
   W *kcross, *vcross;          // [Ld][max_src][d]
   Partial* part;               // [grid][rows]
-  int* y;                      // [max_tgt + 1]: y_0 = BOS, then the draft / solution
   DecState* st;
   pd_trace_step* trace;        // [max_tgt]
   int* trace_tok;              // [max_tgt][max_tgt]
@@ -206,18 +207,9 @@ __device__ __forceinline__ void tl_dump() {
 __device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
-__device__ __forceinline__ unsigned atom_acq_rel_add(unsigned* p, unsigned v) {
-  unsigned old;
-  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v)
-               : "memory");
-  return old;
-}
-__device__ __forceinline__ void st_release_u32(unsigned* p, unsigned v) {
-  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
 
-// Bar words: [0] arrival counter (only grows), [1] abort flag, [2] release word of the
-// commit barrier.  Spin until *word >= target; give up after kWaitNs, raising the abort flag
+// Bar words: [0] arrival counter (only grows), [1] abort flag (words 2, 3 spare).  Spin until
+// *word >= target; give up after kWaitNs, raising the abort flag
 // and PD_ETIMEOUT, so that a broken schedule ends the kernel instead of hanging the GPU.
 // The abort flag and the clock are looked at every 32nd poll only: a poll is then a single
 // load, and the barrier is released one round trip after its last arrival.
@@ -270,34 +262,6 @@ __device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, in
 }
 __device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, int* status) {
   return grid_barrier(bar, target, status, [] {});
-}
-
-// A barrier whose last arriving CTA runs `last()` before anybody is released: it sees every
-// CTA's writes (acq_rel arrival) and its own writes are released with the release word.
-// Folds the fixed-point commit into the LM-head barrier.  Returns false on abort.
-template <typename F>
-__device__ __forceinline__ bool grid_barrier_last(unsigned* bar, unsigned& target, int* status,
-                                                  F&& last) {
-  __shared__ int s_ok, s_last;
-  __syncthreads();
-  target += gridDim.x;
-  TL(3); TLG(5);
-  if (threadIdx.x == 0) {
-    const unsigned old = atom_acq_rel_add(bar, 1u);
-    s_last = old + 1u == target;
-    s_ok = 1;
-  }
-  __syncthreads();
-  if (s_last) {
-    last();
-    __syncthreads();
-    if (threadIdx.x == 0) st_release_u32(bar + 2, target);
-  } else if (threadIdx.x == 0) {
-    s_ok = spin_until(bar, bar + 2, target, status);
-  }
-  TL_NEXT(); TL(0); TLG(4);
-  __syncthreads();
-  return s_ok != 0;
 }
 
 // Ask L2 to fetch [p, p + bytes) ahead of use (no data returns to the SM).  The weights of a
@@ -473,6 +437,15 @@ __device__ __forceinline__ uint4 ld_act16(const void* p) {
   return v;
 }
 
+// Four consecutive elements p[0..3] as floats, one vector load (p is 4-element aligned: every
+// tensor of the weight blob and every shared-memory copy starts at a multiple of 256 elements).
+__device__ __forceinline__ float4 get4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 get4(const __nv_bfloat16* p) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);      // bf16 = the high half of a float
+  return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                     __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+}
+
 // LayerNorm of a row held as float4 v[i] = elements lane*4 + 128*i: mean and biased variance
 // from per-lane sums in ascending i, then fixed butterflies.
 template <typename W>
@@ -497,10 +470,11 @@ __device__ __forceinline__ void ln_regs(float4 (&v)[kMaxRowRegs], int nI, int K,
   for (int i = 0; i < kMaxRowRegs; ++i) {
     if (i < nI) {
       const int k = lane * 4 + 128 * i;
-      v[i].x = (v[i].x - mean) * rstd * to_f(g[k]) + to_f(b[k]);
-      v[i].y = (v[i].y - mean) * rstd * to_f(g[k + 1]) + to_f(b[k + 1]);
-      v[i].z = (v[i].z - mean) * rstd * to_f(g[k + 2]) + to_f(b[k + 2]);
-      v[i].w = (v[i].w - mean) * rstd * to_f(g[k + 3]) + to_f(b[k + 3]);
+      const float4 gk = get4(g + k), bk = get4(b + k);
+      v[i].x = (v[i].x - mean) * rstd * gk.x + bk.x;
+      v[i].y = (v[i].y - mean) * rstd * gk.y + bk.y;
+      v[i].z = (v[i].z - mean) * rstd * gk.z + bk.z;
+      v[i].w = (v[i].w - mean) * rstd * gk.w + bk.w;
     }
   }
 }
@@ -514,10 +488,6 @@ __device__ __forceinline__ void put4(__nv_bfloat16* xs, float4 v) {
   *reinterpret_cast<uint2*>(xs) = u;
 }
 
-template <typename W>
-__device__ __forceinline__ float4 get4(const W* p) {
-  return make_float4(to_f(p[0]), to_f(p[1]), to_f(p[2]), to_f(p[3]));
-}
 
 // Stage rows m0..m0+mt of the GEMM input into shared memory (one warp per row, each element
 // loaded once into registers).
