@@ -59,9 +59,9 @@ def main(argv=None):
     nph = 8 * spec.n_dec_layers + 1
     G = torch.cuda.get_device_properties(0).multi_processor_count    # one CTA per SM
     buf = torch.zeros(K_TL * G * MARKS, dtype=torch.int64, device="cuda")
-    # interval 0 is the start; the decode loop's first barrier opens interval 1, then every
-    # pass has nph intervals
-    assert lib.pd_debug_set_tl(buf.data_ptr(), 1 + args.pass_index * nph) == 0
+    # interval 0 runs from the kernel start to the first barrier (phase 0 of pass 0); every
+    # pass has nph intervals, the first of which also holds the commit of the pass before
+    assert lib.pd_debug_set_tl(buf.data_ptr(), args.pass_index * nph) == 0
     dec.encode(src)
     for _ in range(3):
         buf.zero_()
