@@ -37,8 +37,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
 # ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel sources whose
 # SHA-256 is recorded here; any other source reports traffic null.
-DRAM_BYTES_PER_PASS = 12.39e6
-DRAM_SOURCES_SHA256 = "479e0472a9d0c0fc5e7d2e1417566c7a5849010a5a53c7bfb81fbe686d611189"
+DRAM_BYTES_PER_PASS = 14.86e6
+DRAM_SOURCES_SHA256 = "a4c054c6dd124bdea4beb9ce6ea3b4573e1b69edb7667fc8f4b9dba3106027ee"
 
 
 def kernel_sources_sha256() -> str:
