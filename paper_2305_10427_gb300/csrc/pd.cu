@@ -273,6 +273,14 @@ __device__ void prefetch_phase(const KParams<W>& P, int ph) {
   }
 }
 
+// The weights a pass reads first (phases 0 and 2), asked from L2 when the pass starts; every
+// later GEMM phase's weights, the LM head's table included, are asked three phases ahead.
+template <typename W>
+__device__ void prefetch_pass_start(const KParams<W>& P) {
+  prefetch_phase(P, 0);
+  prefetch_phase(P, 2);
+}
+
 template <typename W>
 __device__ __forceinline__ GemmArgs<W>& smem_args() {
   __shared__ GemmArgs<W> s;
@@ -281,7 +289,7 @@ __device__ __forceinline__ GemmArgs<W>& smem_args() {
 
 // One decoder pass over M rows followed by the LM head, as a loop over phases separated by
 // grid barriers.  The arguments of the next GEMM phase are written to shared memory by one
-// thread while its CTA waits at the barrier, and the weights two phases ahead are requested
+// thread while its CTA waits at the barrier, and the weights three phases ahead are requested
 // from L2 there, so that neither is on the chain of dependent phases.
 template <typename W>
 __device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, float* logits,
@@ -295,9 +303,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, f
   GemmArgs<W>& ga = smem_args<W>();
   const int nph = 8 * D.Ld + 1;
   if (threadIdx.x == 32) gemm_args(P, 0, M, pos0, tok, logits, ga);
-  prefetch_phase(P, 0);
-  prefetch_phase(P, 2);
-  prefetch_phase(P, nph - 1);
+  prefetch_pass_start(P);
   __syncthreads();
   for (int ph = 0; ph < nph; ++ph) {
     const bool attn = is_attn_phase(ph, nph);
@@ -388,15 +394,16 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
     }
   }
   if (tid == 0) {
+    DecState st = ss;                              // decisions on a register copy
     int c = 0;                                     // leading positions equal to the old draft
     while (c < blk && ntok[c] == sy[i + c]) ++c;
     const int stop = c == blk;
     int eos_idx = -1;
     for (int r = 0; r < blk; ++r)
       if (ntok[r] == D.eos) { eos_idx = r; break; }
-    ss.k = ss.k + 1;
-    const int n_it = ss.n_iters + 1;
-    ss.n_iters = n_it;
+    st.k = st.k + 1;
+    const int n_it = st.n_iters + 1;
+    st.n_iters = n_it;
     if (t < D.max_tgt) {
       if (blockIdx.x == 0) {
         pd_trace_step row;
@@ -404,49 +411,50 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
         row.stop = stop; row.eos_idx = eos_idx;
         B.trace[t] = row;
       }
-      ss.n_trace = t + 1;
+      st.n_trace = t + 1;
     }
     if (s_nan) {
-      ss.status = PD_ENAN; ss.n_y = i - 1; ss.done = 1;
+      st.status = PD_ENAN; st.n_y = i - 1; st.done = 1;
     } else {
       // the block is solved: StopC, the pass cap, or (accepted-prefix rule) the first c + 1
       // new tokens exact with c + 1 >= blk
-      if (stop || ss.k >= blk || (ss.stop_rule == PD_STOP_PREFIX && c + 1 >= blk)) {
-        const bool one_pos = ss.method == PD_GREEDY || ss.ar_tail;
+      if (stop || st.k >= blk || (st.stop_rule == PD_STOP_PREFIX && c + 1 >= blk)) {
+        const bool one_pos = st.method == PD_GREEDY || st.ar_tail;
         if (one_pos) {
-          const bool eos_ends = ss.ar_tail ? true : (ss.stop_at_eos != 0);
-          if (eos_ends && ntok[0] == D.eos) { ss.n_y = i; ss.done = 1; }
-        } else if (ss.method == PD_HYBRID_GS_JACOBI && eos_idx >= 0) {
-          ss.n_y = i + eos_idx;                    // through the EOS (Algorithm 3)
-          ss.done = 1;
+          const bool eos_ends = st.ar_tail ? true : (st.stop_at_eos != 0);
+          if (eos_ends && ntok[0] == D.eos) { st.n_y = i; st.done = 1; }
+        } else if (st.method == PD_HYBRID_GS_JACOBI && eos_idx >= 0) {
+          st.n_y = i + eos_idx;                    // through the EOS (Algorithm 3)
+          st.done = 1;
         }
-        if (!ss.done) {
+        if (!st.done) {
           const int ni = i + blk;
-          if (ss.method == PD_HYBRID_GS_JACOBI && !ss.ar_tail && ni > ss.h) {
-            ss.ar_tail = 1;                        // greedy tail up to max_len
-            ss.b_eff = 1;
-            ss.m_eff = ss.max_len;
+          if (st.method == PD_HYBRID_GS_JACOBI && !st.ar_tail && ni > st.h) {
+            st.ar_tail = 1;                        // greedy tail up to max_len
+            st.b_eff = 1;
+            st.m_eff = st.max_len;
           }
-          if (ni > ss.m_eff) {
-            ss.done = 1;
-            ss.n_y = ss.m_eff;
-            s_scan = (ss.method == PD_JACOBI || ss.method == PD_GS_JACOBI) && ss.stop_at_eos;
+          if (ni > st.m_eff) {
+            st.done = 1;
+            st.n_y = st.m_eff;
+            s_scan = (st.method == PD_JACOBI || st.method == PD_GS_JACOBI) && st.stop_at_eos;
           } else {
-            ss.i = ni;
-            const int rest = ss.m_eff - ni + 1;
-            ss.blk = ss.b_eff < rest ? ss.b_eff : rest;
-            ss.k = 0;
+            st.i = ni;
+            const int rest = st.m_eff - ni + 1;
+            st.blk = st.b_eff < rest ? st.b_eff : rest;
+            st.k = 0;
           }
         }
       }
       // the pass budget, and a hard cap no correct schedule reaches (at most m passes for the
       // parallel part plus max_len for a greedy tail): the loop can never run away
-      if (!ss.done && ((ss.max_passes > 0 && n_it >= ss.max_passes) || n_it > 2 * ss.max_len + 2)) {
-        ss.status = PD_ENOTCONV;
-        ss.n_y = ss.i - 1;
-        ss.done = 1;
+      if (!st.done && ((st.max_passes > 0 && n_it >= st.max_passes) || n_it > 2 * st.max_len + 2)) {
+        st.status = PD_ENOTCONV;
+        st.n_y = st.i - 1;
+        st.done = 1;
       }
     }
+    ss = st;
   }
   __syncthreads();
   for (int r = tid; r < blk; r += blockDim.x) sy[i + r] = ntok[r];   // y_{i:i+blk} <- new
