@@ -273,12 +273,13 @@ __device__ void prefetch_phase(const KParams<W>& P, int ph) {
   }
 }
 
-// The weights a pass reads first (phases 0 and 2), asked from L2 when the pass starts; every
-// later GEMM phase's weights, the LM head's table included, are asked three phases ahead.
+// The weights a pass reads first (phases 0 and 2) and the LM head's table, asked from L2 when
+// the pass starts (the other phases' weights are asked three phases ahead).
 template <typename W>
 __device__ void prefetch_pass_start(const KParams<W>& P) {
   prefetch_phase(P, 0);
   prefetch_phase(P, 2);
+  prefetch_phase(P, 8 * P.D.Ld);
 }
 
 template <typename W>
