@@ -37,8 +37,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
 # ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel sources whose
 # SHA-256 is recorded here; any other source reports traffic null.
-DRAM_BYTES_PER_PASS = 14.86e6
-DRAM_SOURCES_SHA256 = "a4c054c6dd124bdea4beb9ce6ea3b4573e1b69edb7667fc8f4b9dba3106027ee"
+DRAM_BYTES_PER_PASS = 15.11e6
+DRAM_SOURCES_SHA256 = "5116511b50002a0d4a707116b029cdb49564192eb524701b21336d45bca248c7"
 
 
 def kernel_sources_sha256() -> str:
