@@ -10,10 +10,14 @@
   from random initial drafts, in at most m passes.
 * Structural identities: GS-Jacobi with b = 1 is greedy pass for pass; Jacobi is GS-Jacobi
   with b = m; one teacher-forced pass over the greedy output reproduces it (Eq. 4, f = 0).
+* Full per-pass traces on the planted structures equal the hand-derived ones of
+  tests/golden/planted_traces.txt (StopC flags, unchanged-prefix counts, block starts, EOS
+  index, both stop rules, hybrid EOS exit and greedy tail).
 * Planted mistakes in the loops are caught.
 """
 import itertools
 import math
+import os
 
 import numpy as np
 import pytest
@@ -87,6 +91,46 @@ def test_trace_rows_of_a_chain_block():
     assert [t.stop for t in r.trace] == [False] * 4
     assert all(t.block_start == 1 and t.block_len == 4 for t in r.trace)
     assert r.trace[-1].tokens == r.tokens
+
+
+GOLDEN_TRACES = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden",
+                             "planted_traces.txt")
+
+
+def _golden_trace_cases():
+    cases = []
+    for line in open(GOLDEN_TRACES):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        if line.startswith("case "):
+            f = line.split()
+            cases.append(dict(kv.split("=") for kv in f[3:]))
+            cases[-1].update(structure=f[1], method=f[2], header=line[5:], rows=[])
+        else:
+            cases[-1]["rows"].append(tuple(int(v) for v in line.split()))
+    return cases
+
+
+@pytest.mark.parametrize("case", _golden_trace_cases(), ids=lambda c: c["header"])
+def test_golden_planted_traces(case):
+    eos_at = int(case["eos"]) if "eos" in case else None
+    step = {"position_only": position_only(eos_at), "chain": chain,
+            "skip_chain": skip_chain}[case["structure"]]
+    m, b, rule = int(case["m"]), int(case["b"]), case["rule"]
+    if case["method"] == "jacobi":
+        r = od.jacobi(step, m, stop_at_eos=False, stop_rule=rule)
+    elif case["method"] == "gs_jacobi":
+        r = od.gs_jacobi(step, m, b, stop_at_eos=False, stop_rule=rule)
+    else:
+        r = od.hybrid_gs_jacobi(step, m, b, h=int(case["h"]) if "h" in case else None,
+                                stop_rule=rule)
+    got = [(t.step, t.block_start, t.block_len, t.n_converged, int(t.stop), t.eos_idx)
+           for t in r.trace]
+    assert got == case["rows"]
+    assert r.n_iters == len(case["rows"])
+    assert len(r.tokens) == int(case["tokens"])
+    assert r.tokens == od.greedy(step, m, stop_at_eos=case["method"] == "hybrid_gs_jacobi").tokens
 
 
 def test_hybrid_eos_and_tail():
