@@ -37,6 +37,11 @@ struct KParams {
   int32_t* out_info;        // {n_y, n_iters, status, n_trace}
 };
 
+// Dynamic shared memory of the decode / encode kernels (byte offsets): xs, the staged GEMM
+// input rows (8 rows x max(d, f) in the weight type); part, the LM head's per-warp argmax
+// partials; scratch, the attention phase's per-warp scaled query and scores; commit, the new
+// block tokens, their probabilities and this CTA's copy of y_0..y_m (3 x (max_tgt + 1) ints);
+// ln, the copied LayerNorm vectors and biases (ln_bytes, possibly 0).
 struct SmemLayout {
   size_t xs, part, scratch, commit, ln, ln_bytes, total;
 };
