@@ -205,6 +205,23 @@ def _bad_scale(orig_attention):
     return f
 
 
+def _wrap_attention(change):
+    """Plant a mistake in the arguments every attention call receives."""
+    def patch(mp):
+        orig = om.attention
+
+        def f(*args):
+            return orig(*change(*args))
+        mp.setattr(om, "attention", f)
+    return patch
+
+
+def _wrap_method(name, make):
+    def patch(mp):
+        mp.setattr(om.Model, name, make(getattr(om.Model, name)))
+    return patch
+
+
 MUTATIONS = {
     "no causal mask": lambda mp: mp.setattr(om, "attention", _no_causal_mask(om.attention)),
     "sin/cos swapped": lambda mp: mp.setattr(
@@ -216,6 +233,24 @@ MUTATIONS = {
     "query perturbed": lambda mp: mp.setattr(om, "attention", _bad_scale(om.attention)),
     "relu for silu": lambda mp: mp.setattr(
         om, "activation", (lambda orig: lambda x, k: orig(x, synth.ACT_RELU))(om.activation)),
+    "keys and values swapped": _wrap_attention(
+        lambda xq, xkv, wq, bq, wk, bk, wv, bv, wo, bo, h, c:
+        (xq, xkv, wq, bq, wv, bv, wk, bk, wo, bo, h, c)),
+    "output projection transposed": _wrap_attention(
+        lambda xq, xkv, wq, bq, wk, bk, wv, bv, wo, bo, h, c:
+        (xq, xkv, wq, bq, wk, bk, wv, bv, wo.T, bo, h, c)),
+    "heads merged into one": _wrap_attention(
+        lambda xq, xkv, wq, bq, wk, bk, wv, bv, wo, bo, h, c:
+        (xq, xkv, wq, bq, wk, bk, wv, bv, wo, bo, 1, c)),
+    "embedding not scaled by sqrt(d)": _wrap_method(
+        "embed", lambda orig: lambda self, ids, side:
+        orig(self, ids, side) - self.w["embed"][np.asarray(ids)] * (math.sqrt(self.s.d_model) - 1)),
+    "positions shifted by one": _wrap_method(
+        "embed", lambda orig: lambda self, ids, side:
+        orig(self, ids, side) - om.sinusoid(np.arange(len(ids)), self.s.d_model)
+        + om.sinusoid(np.arange(1, len(ids) + 1), self.s.d_model)),
+    "cross-attention to the decoder states": _wrap_method(
+        "_cross_attn", lambda orig: lambda self, x, mem, p: orig(self, x, x, p)),
 }
 
 
