@@ -48,3 +48,24 @@ def test_pass_bytes_model():
     got = bench.pass_bytes(spec, L_keys=10, n_src=7, rows=5)
     assert got == 2 * (weights + L * 2 * d * (10 + 7) + L * 2 * d * 5)
     assert 103e6 < 2 * weights < 104e6
+
+
+def test_reference_arm_prints_one_contract_line():
+    """bench.py --impl reference (the CPU oracle arm the driver runs beside the GPU arm)
+    prints exactly one JSON line with the contract's keys."""
+    import json
+    import subprocess
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference",
+                          "--steps", "1", "--warmup", "1"], capture_output=True, text=True,
+                         timeout=600, check=True).stdout.strip().splitlines()
+    assert len(out) == 1
+    line = json.loads(out[0])
+    for k in ("impl", "metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+              "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config",
+              "cpu_baseline", "e2e"):
+        assert k in line, k
+    assert line["impl"] == "reference" and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"]["value"] == line["value"]
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
