@@ -62,7 +62,7 @@ struct CommitMem {
   DecState* st;
   int* r0;
   int* y;                   // [max_batch][max_tgt + 1]
-  int* misc;                // [0] rows of the current pass, [1] scan request flags
+  int* misc;                // [0] rows of the current pass
 };
 __host__ __device__ inline size_t commit_bytes(const Dims& D) {
   return (size_t)D.rows * 9 * 4 + (size_t)D.max_batch * (sizeof(DecState) + 4) +
