@@ -665,6 +665,9 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
   const EmbedTabs<W> T = embed_tabs(P);
   const bool pre = D.pre_ln != 0;
   const int n = P.n_src;
+  const CommitMem cm = commit_mem(D, smem + SL.commit);
+  for (int m = threadIdx.x; m < n; m += blockDim.x) cm.rpos[m] = m;   // source positions
+  __syncthreads();
 
   for (int l = 0; l < D.Le; ++l) {
     const EncLayerW<W>& L = mw.enc[l];
@@ -680,7 +683,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     GemmArgs<W> g{};
     g.M = n; g.N = 3 * D.d; g.K = D.d;
     if (l == 0) {
-      g.emb_tok = P.enc_tok; g.x_store = B.ra;            // positions 0..n-1
+      g.emb_tok = P.enc_tok; g.emb_pos = cm.rpos; g.x_store = B.ra;   // positions 0..n-1
       if (pre) { g.ln_a_g = mw.enc_lne_g; g.ln_a_b = mw.enc_lne_b; g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
     } else {
       g.x_src = B.ra;

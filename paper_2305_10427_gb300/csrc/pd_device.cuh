@@ -305,7 +305,7 @@ struct GemmArgs {
   const float* x_src;
   const W* xw_src;          // input rows already rounded to W (plain copy; instead of x_src)
   const int* emb_tok;
-  const int* emb_pos;       // per-row positions (nullptr: row m is at position m)
+  const int* emb_pos;       // per-row positions of the embedded rows
   const W *ln_a_g, *ln_a_b;
   float* x_store;
   const W *ln_b_g, *ln_b_b;
@@ -316,9 +316,9 @@ struct GemmArgs {
   W* out_w;                 // [M][ld] for ACT
   int ld;
   const float* resid;       // [M][ld]
-  W *kdst, *vdst;           // QKV: cache rows (slot[m], or m); KVCROSS: cross caches
+  W *kdst, *vdst;           // QKV: cache rows slot[m]; KVCROSS: cross caches
   float *kdst_f, *vdst_f;   // QKV into fp32 buffers (encoder)
-  const int* slot;          // QKV: per-row cache slots (nullptr: m)
+  const int* slot;          // QKV into kdst / vdst: per-row cache slots
   Partial* part;            // ARGMAX: [grid][rows_ld]
   int part_ld;
   // How the phase is divided over the grid (gemm_plan): column groups, K-steps per warp,
@@ -551,7 +551,7 @@ __device__ void stage_x(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims&
     if (g.emb_tok != nullptr) {
       int t = g.emb_tok[m];
       t = t < 0 ? 0 : (t >= D.V ? D.V - 1 : t);
-      const int p = g.emb_pos != nullptr ? g.emb_pos[m] : m;
+      const int p = g.emb_pos[m];
       const W* er = T.E + (size_t)t * K;
 #pragma unroll
       for (int i = 0; i < kMaxRowRegs; ++i) {
@@ -712,7 +712,7 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
             g.out[(size_t)m * D.d + cc] = v;
           } else if (g.kdst != nullptr) {
             W* dst = which == 1 ? g.kdst : g.vdst;
-            dst[(size_t)(g.slot != nullptr ? g.slot[m] : m) * D.d + cc] = from_f<W>(v);
+            dst[(size_t)g.slot[m] * D.d + cc] = from_f<W>(v);
           } else {
             float* dst = which == 1 ? g.kdst_f : g.vdst_f;
             dst[(size_t)m * D.d + cc] = v;
