@@ -71,6 +71,8 @@ typedef struct {
   float ln_eps;
   int max_src_len;   /* capacity: longest source sentence pd_encode accepts */
   int max_tgt_len;   /* capacity: largest max_len pd_decode accepts */
+  int max_batch;     /* capacity: sentences one pd_encode_batch / pd_decode_batch carries,
+                        0 or 1..64 (0 = 1); each needs its own key/value caches */
 } pd_config;
 
 typedef struct pd_ctx pd_ctx;
@@ -148,6 +150,39 @@ pd_status pd_decode(pd_ctx* ctx, const pd_decode_params* p, int32_t* y, int* n_y
  * and d_info[4] = {n_y, n_iters, status, n_trace}.  Parameters are checked on the host. */
 pd_status pd_decode_device(pd_ctx* ctx, const pd_decode_params* p, int32_t* d_y,
                            int32_t* d_info);
+
+/* Batched serving (several independent sentences decoded together; the paper decodes one
+ * sentence at a time, Section 4.1, and every result below is exactly that sentence's alone).
+ *
+ * pd_encode_batch: run the encoder for sentences s = 0..n_sent-1 (1 <= n_sent <= max_batch),
+ * sentence s being src[offsets[s] .. offsets[s+1]) (host int32; offsets[0] = 0, every length in
+ * [1, max_src_len], ids in [0, vocab)), caching each one's cross-attention keys and values in
+ * slot s.  Synchronous.  pd_encode is pd_encode_batch of one sentence. */
+pd_status pd_encode_batch(pd_ctx* ctx, const int32_t* src, const int32_t* offsets, int n_sent);
+
+/* As pd_encode_batch with the ids in device memory (d_src) and offsets on the host;
+ * asynchronous on the context stream (ids are not range-checked). */
+pd_status pd_encode_batch_device(pd_ctx* ctx, const int32_t* d_src, const int32_t* offsets,
+                                 int n_sent);
+
+/* Decode the n_sent sentences of the last pd_encode_batch together: one decoder pass carries
+ * the current block of every sentence that is not finished (at most 512 rows in all: the sum
+ * over sentences of min(block size, max_len) must fit), each sentence with its own block
+ * position, convergence test, EOS handling and pass count, as pd_decode would run it alone.
+ * p gives the method and its parameters for all sentences; max_len (host int32[n_sent], or
+ * NULL for p->max_len everywhere) the known length m of each.  Outputs (host): y[s * y_ld ..]
+ * = sentence s's tokens (y_ld >= its max_len), n_y[s], n_iters[s] = passes in which sentence s
+ * took part.  No trace.  Synchronous.  Returns PD_OK, or the status of the first sentence that
+ * failed (outputs are filled for all). */
+pd_status pd_decode_batch(pd_ctx* ctx, const pd_decode_params* p, int n_sent,
+                          const int32_t* max_len, int32_t* y, int y_ld, int32_t* n_y,
+                          int32_t* n_iters);
+
+/* As pd_decode_batch, asynchronous on the context stream, outputs in device memory:
+ * d_y[n_sent][y_ld] and d_info[n_sent][4] = {n_y, n_iters, status, n_trace}. */
+pd_status pd_decode_batch_device(pd_ctx* ctx, const pd_decode_params* p, int n_sent,
+                                 const int32_t* max_len, int32_t* d_y, int y_ld,
+                                 int32_t* d_info);
 
 /* Test-only: teacher-forced logits of one decoder pass over the input tokens y_in[0..len)
  * at positions 0..len-1 (row t scores position t+1, Eq. 1) for the sentence last encoded.

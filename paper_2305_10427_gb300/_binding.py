@@ -28,7 +28,8 @@ STOP_RULES = {"paper": 0, "prefix": 1}      # pd_stop_rule: Eq. 5 StopC, accepte
 EXPORTED = ("pd_weights_nbytes", "pd_create", "pd_export_weights", "pd_encode",
             "pd_encode_device", "pd_decode", "pd_decode_device", "pd_debug_logits",
             "pd_debug_logits_static", "pd_debug_wait_timeout", "pd_stream", "pd_launch_count",
-            "pd_last_error", "pd_destroy")
+            "pd_last_error", "pd_destroy", "pd_encode_batch", "pd_encode_batch_device",
+            "pd_decode_batch", "pd_decode_batch_device")
 
 
 class PdError(RuntimeError):
@@ -43,7 +44,7 @@ class _Config(ctypes.Structure):
                                             "learned_pos", "max_pos", "dtype", "pad_id",
                                             "eos_id", "bos_id")] + \
               [("ln_eps", ctypes.c_float), ("max_src_len", ctypes.c_int),
-               ("max_tgt_len", ctypes.c_int)]
+               ("max_tgt_len", ctypes.c_int), ("max_batch", ctypes.c_int)]
 
 
 class _DecodeParams(ctypes.Structure):
@@ -86,6 +87,14 @@ def load_library() -> ctypes.CDLL:
     lib.pd_decode.restype = I
     lib.pd_decode_device.argtypes = [P, ctypes.POINTER(_DecodeParams), P, P]
     lib.pd_decode_device.restype = I
+    lib.pd_encode_batch.argtypes = [P, pi32, pi32, I]
+    lib.pd_encode_batch.restype = I
+    lib.pd_encode_batch_device.argtypes = [P, P, pi32, I]
+    lib.pd_encode_batch_device.restype = I
+    lib.pd_decode_batch.argtypes = [P, ctypes.POINTER(_DecodeParams), I, pi32, pi32, I, pi32, pi32]
+    lib.pd_decode_batch.restype = I
+    lib.pd_decode_batch_device.argtypes = [P, ctypes.POINTER(_DecodeParams), I, pi32, P, I, P]
+    lib.pd_decode_batch_device.restype = I
     lib.pd_debug_logits.argtypes = [P, pi32, I, ctypes.POINTER(ctypes.c_float)]
     lib.pd_debug_logits.restype = I
     lib.pd_debug_logits_static.argtypes = [P, pi32, I, ctypes.POINTER(ctypes.c_float)]
@@ -125,14 +134,16 @@ class Config:
     ln_eps: float = 1e-5
     max_src_len: int = 128
     max_tgt_len: int = 256
+    max_batch: int = 0
 
     @classmethod
-    def from_spec(cls, spec, max_src_len: int, max_tgt_len: int, pad_id=1, eos_id=0, bos_id=2):
+    def from_spec(cls, spec, max_src_len: int, max_tgt_len: int, pad_id=1, eos_id=0, bos_id=2,
+                  max_batch: int = 0):
         """Build from any object carrying the model fields (d_model, n_heads, ...)."""
         return cls(spec.d_model, spec.n_heads, spec.d_ff, spec.n_enc_layers, spec.n_dec_layers,
                    spec.vocab, spec.activation, bool(spec.pre_ln), bool(spec.learned_pos),
                    spec.max_pos, spec.dtype, pad_id, eos_id, bos_id, spec.ln_eps, max_src_len,
-                   max_tgt_len)
+                   max_tgt_len, max_batch)
 
     def _c(self) -> _Config:
         c = _Config()
@@ -190,6 +201,48 @@ class Decoder:
     def encode_device(self, d_src: int, n_src: int) -> None:
         self._check(self._lib.pd_encode_device(self._h, ctypes.c_void_p(d_src), int(n_src)),
                     "pd_encode_device")
+
+    @staticmethod
+    def batch_offsets(sents):
+        """Concatenated ids and the offsets array of pd_encode_batch."""
+        arrs = [np.ascontiguousarray(s, dtype=np.int32) for s in sents]
+        offs = np.zeros(len(arrs) + 1, dtype=np.int32)
+        offs[1:] = np.cumsum([a.size for a in arrs])
+        return np.concatenate(arrs), offs
+
+    def encode_batch(self, sents) -> None:
+        src, offs = self.batch_offsets(sents)
+        self._check(self._lib.pd_encode_batch(self._h, _i32p(src), _i32p(offs), len(offs) - 1),
+                    "pd_encode_batch")
+
+    def encode_batch_device(self, d_src: int, offsets: np.ndarray) -> None:
+        offs = np.ascontiguousarray(offsets, dtype=np.int32)
+        self._check(self._lib.pd_encode_batch_device(self._h, ctypes.c_void_p(d_src), _i32p(offs),
+                                                     offs.size - 1), "pd_encode_batch_device")
+
+    def decode_batch(self, method: str, max_len, b: int = 1, h: int = 0,
+                     stop_at_eos: bool = True, max_passes: int = 0,
+                     stop_rule: str = "paper") -> List["DecodeResult"]:
+        """Decode the sentences of the last encode_batch together; max_len: one value per
+        sentence."""
+        ml = np.ascontiguousarray(max_len, dtype=np.int32)
+        n = ml.size
+        p = self.params(method, int(ml.max()), b, h, stop_at_eos, max_passes, stop_rule)
+        y_ld = int(ml.max())
+        y = np.zeros((n, y_ld), dtype=np.int32)
+        n_y = np.zeros(n, dtype=np.int32)
+        n_it = np.zeros(n, dtype=np.int32)
+        self._check(self._lib.pd_decode_batch(self._h, ctypes.byref(p), n, _i32p(ml), _i32p(y), y_ld,
+                                              _i32p(n_y), _i32p(n_it)), "pd_decode_batch")
+        return [DecodeResult([int(t) for t in y[s, :n_y[s]]], int(n_it[s])) for s in range(n)]
+
+    def decode_batch_device(self, p: _DecodeParams, max_len: np.ndarray, d_y: int, y_ld: int,
+                            d_info: int) -> None:
+        ml = np.ascontiguousarray(max_len, dtype=np.int32)
+        self._check(self._lib.pd_decode_batch_device(self._h, ctypes.byref(p), ml.size, _i32p(ml),
+                                                     ctypes.c_void_p(d_y), int(y_ld),
+                                                     ctypes.c_void_p(d_info)),
+                    "pd_decode_batch_device")
 
     @staticmethod
     def params(method: str, max_len: int, b: int = 1, h: int = 0, stop_at_eos: bool = True,

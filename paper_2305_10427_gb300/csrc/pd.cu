@@ -16,6 +16,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <algorithm>
 #include <vector>
 
 #include "pd.h"
@@ -28,23 +29,63 @@ struct KParams {
   Dims D;
   const ModelW<W>* mw;      // device copy of the weight-pointer table
   Bufs<W> B;
-  int n_src;                // encoder length (cross-attention keys)
+  int n_src;                // encode: source length
+  int enc_slot;             // encode: cache slot of the sentence (0 for pd_encode)
   const int* enc_tok;       // encoder input ids (device)
-  int debug_len;            // > 0: one teacher-forced pass over dbg_tok, logits out
+  int debug_len;            // > 0: one teacher-forced pass over dbg_tok (slot 0), logits out
   float* logits;            // [debug_len][V]
-  DecState init;            // method, b, max_len, h, stop_at_eos, max_passes, stop_rule
-  int32_t* out_y;           // [max_len]
-  int32_t* out_info;        // {n_y, n_iters, status, n_trace}
+  DecState init;            // method, b, h, stop_at_eos, max_passes, stop_rule (all sentences)
+  int n_sent;               // decode: sentences, slots 0..n_sent-1
+  int n_src_s[kMaxBatch];   // decode: source length of each sentence
+  int max_len_s[kMaxBatch]; // decode: max_len (the known m of Jacobi / GS-Jacobi) of each
+  int32_t* out_y;           // [n_sent][out_ld]
+  int out_ld;
+  int32_t* out_info;        // [n_sent][4] = {n_y, n_iters, status, n_trace}
 };
 
 // Dynamic shared memory of the decode / encode kernels (byte offsets): xs, the staged GEMM
 // input rows (8 rows x max(d, f) in the weight type); part, the LM head's per-warp argmax
-// partials; scratch, the attention phase's per-warp scaled query and scores; commit, the new
-// block tokens, their probabilities and this CTA's copy of y_0..y_m (3 x (max_tgt + 1) ints);
-// ln, the copied LayerNorm vectors and biases (ln_bytes, possibly 0).
+// partials; scratch, the attention phase's per-warp scaled query and scores; commit, the
+// decoding state of this CTA (see CommitMem); ln, the copied LayerNorm vectors and biases
+// (ln_bytes, possibly 0).
 struct SmemLayout {
   size_t xs, part, scratch, commit, ln, ln_bytes, total;
 };
+
+// The commit region: per pass row r (at most D.rows) its new token (-1 for a NaN row) and
+// probability, and the row's description (input token, position, self-attention cache slot,
+// first slot of its sentence, keys it attends, first cross key row and cross key count); per
+// sentence its decoding state, its first row in the pass and y_0..y_m.
+struct CommitMem {
+  int *ntok, *rtok, *rpos, *rslot, *rsb, *rkn, *rxb, *rxn;
+  float* nprob;
+  DecState* st;
+  int* r0;
+  int* y;                   // [max_batch][max_tgt + 1]
+  int* misc;                // [0] rows of the current pass
+};
+__host__ __device__ inline size_t commit_bytes(const Dims& D) {
+  return (size_t)D.rows * 9 * 4 + (size_t)D.max_batch * (sizeof(DecState) + 4) +
+         (size_t)D.max_batch * (D.max_tgt + 1) * 4 + 64;
+}
+__device__ __forceinline__ CommitMem commit_mem(const Dims& D, unsigned char* base) {
+  CommitMem c;
+  int* p = reinterpret_cast<int*>(base);
+  c.ntok = p; p += D.rows;
+  c.rtok = p; p += D.rows;
+  c.rpos = p; p += D.rows;
+  c.rslot = p; p += D.rows;
+  c.rsb = p; p += D.rows;
+  c.rkn = p; p += D.rows;
+  c.rxb = p; p += D.rows;
+  c.rxn = p; p += D.rows;
+  c.nprob = reinterpret_cast<float*>(p); p += D.rows;
+  c.st = reinterpret_cast<DecState*>(p); p += D.max_batch * (int)(sizeof(DecState) / 4);
+  c.r0 = p; p += D.max_batch;
+  c.y = p; p += D.max_batch * (D.max_tgt + 1);
+  c.misc = p;
+  return c;
+}
 
 // The decoder's small vectors kept in shared memory: the LayerNorm vectors (per layer ln1,
 // ln2, ln3 gamma / beta, and the embedding and final LayerNorms of pre-LN models) when they fit
@@ -62,15 +103,19 @@ __host__ __device__ inline size_t vec_smem_bytes(const Dims& D, size_t wsize) {
   return all <= kVecSmemMax ? all : (ln <= kVecSmemMax ? ln : 0);
 }
 
+constexpr size_t kSmemMax = 227 * 1024;    // dynamic shared memory of one CTA
+
 __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   SmemLayout L;
   const int kmax = D.d > D.f ? D.d : D.f;
   L.xs = 0;
   L.part = L.xs + ((size_t)kMTile * kmax * wsize + 15) / 16 * 16;
   L.scratch = L.part + (size_t)kWarps * 32 * sizeof(Partial);
-  L.commit = L.scratch + (size_t)kWarps * (128 + D.rows + 4) * sizeof(float);
-  L.ln = (L.commit + (size_t)(D.max_tgt + 1) * 3 * sizeof(int) + 64 + 15) / 16 * 16;
-  L.ln_bytes = vec_smem_bytes(D, wsize);
+  L.commit = L.scratch + (size_t)kWarps * (128 + D.max_keys + 4) * sizeof(float);
+  L.ln = (L.commit + commit_bytes(D) + 15) / 16 * 16;
+  // the vector copies are kept only when they fit beside the rest
+  const size_t all = vec_smem_bytes(D, wsize), ln = ln_elems(D) * wsize;
+  L.ln_bytes = L.ln + all <= kSmemMax ? all : (L.ln + ln <= kSmemMax && ln <= kVecSmemMax ? ln : 0);
   L.total = L.ln + L.ln_bytes;
   return L;
 }
@@ -186,11 +231,12 @@ __device__ __forceinline__ bool is_attn_phase(int ph, int nph) {
   return ph < nph - 1 && ((ph & 7) == PH_SELF || (ph & 7) == PH_CROSS);
 }
 
-// Arguments of GEMM phase ph of a pass over M rows at positions pos0.. with input tokens tok;
-// the LM head (ph = 8 Ld) writes raw logits if logits != nullptr, else argmax partials.
+// Arguments of GEMM phase ph of a pass over M rows, row m with input token rtok[m] at position
+// rpos[m] and self-attention cache slot rslot[m]; the LM head (ph = 8 Ld) writes raw logits if
+// logits != nullptr, else argmax partials.
 template <typename W>
-__device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const int* tok,
-                          float* logits, GemmArgs<W>& g) {
+__device__ void gemm_args(const KParams<W>& P, int ph, int M, const int* rtok, const int* rpos,
+                          const int* rslot, float* logits, GemmArgs<W>& g) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
   const ModelW<W>& mw = smem_mw<W>();
@@ -216,7 +262,7 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const in
       // embedding as is.  The embedding is computed in this GEMM's prologue.
       g.N = 3 * D.d; g.K = D.d;
       if (l == 0) {
-        g.emb_tok = tok; g.emb_pos0 = pos0; g.x_store = B.ra;
+        g.emb_tok = rtok; g.emb_pos = rpos; g.x_store = B.ra;
         if (pre) {
           g.ln_a_g = mw.dec_lne_g; g.ln_a_b = mw.dec_lne_b; g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b;
         }
@@ -226,9 +272,9 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, int pos0, const in
         else { g.ln_a_g = mw.dec[l - 1].ln3g; g.ln_a_b = mw.dec[l - 1].ln3b; g.x_store = B.xa; }
       }
       g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
-      g.kdst = B.kself + (size_t)l * D.max_tgt * D.d;
-      g.vdst = B.vself + (size_t)l * D.max_tgt * D.d;
-      g.slot0 = pos0;
+      g.kdst = B.kself + (size_t)l * D.max_batch * D.max_tgt * D.d;
+      g.vdst = B.vself + (size_t)l * D.max_batch * D.max_tgt * D.d;
+      g.slot = rslot;
       break;
     case PH_O:                          // self-attention output + residual
       g.N = D.d; g.K = D.d; g.xw_src = B.att; g.w = L.wo; g.bias = L.bo;
@@ -293,41 +339,46 @@ __device__ __forceinline__ GemmArgs<W>& smem_args() {
   return s;
 }
 
-// One decoder pass over M rows followed by the LM head, as a loop over phases separated by
-// grid barriers.  The arguments of the next GEMM phase are written to shared memory by one
-// thread while its CTA waits at the barrier, and the weights three phases ahead are requested
-// from L2 there, so that neither is on the chain of dependent phases.
+// One decoder pass over the M rows described in the commit region, followed by the LM head, as
+// a loop over phases separated by grid barriers.  The arguments of the next GEMM phase are
+// written to shared memory by one thread while its CTA waits at the barrier, and the weights
+// three phases ahead are requested from L2 there, so that neither is on the chain of dependent
+// phases.
 template <typename W>
-__device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, float* logits,
-                         unsigned& tgt, unsigned char* smem) {
+__device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tgt,
+                         unsigned char* smem) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
+  const CommitMem cm = commit_mem(D, smem + SL.commit);
   const EmbedTabs<W> T = embed_tabs(P);
   GemmArgs<W>& ga = smem_args<W>();
   const int nph = 8 * D.Ld + 1;
-  if (threadIdx.x == 32) gemm_args(P, 0, M, pos0, tok, logits, ga);
+  if (threadIdx.x == 32) gemm_args(P, 0, M, cm.rtok, cm.rpos, cm.rslot, logits, ga);
   prefetch_pass_start(P);
   __syncthreads();
+  const size_t self_ld = (size_t)D.max_batch * D.max_tgt * D.d;
+  const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
   for (int ph = 0; ph < nph; ++ph) {
     const bool attn = is_attn_phase(ph, nph);
     if (attn) {
       const int l = ph >> 3;
       if ((ph & 7) == PH_SELF)
-        attn_phase<W, W>(D, B.q, B.kself + (size_t)l * D.max_tgt * D.d,
-                      B.vself + (size_t)l * D.max_tgt * D.d, B.att, M, pos0, 0, scratch);
+        attn_phase<W, W>(D, B.q, B.kself + l * self_ld, B.vself + l * self_ld, B.att, M,
+                         cm.rsb, cm.rkn, 0, scratch);
       else
-        attn_phase<W, W>(D, B.q, B.kcross + (size_t)l * D.max_src * D.d,
-                      B.vcross + (size_t)l * D.max_src * D.d, B.att, M, -1, P.n_src, scratch);
+        attn_phase<W, W>(D, B.q, B.kcross + l * cross_ld, B.vcross + l * cross_ld, B.att, M,
+                         cm.rxb, cm.rxn, 0, scratch);
     } else {
       gemm_phase<W>(ga, T, D, smem);
     }
     if (ph == nph - 1) break;            // the caller's barrier follows the LM head
     const int next = is_attn_phase(ph + 1, nph) ? ph + 2 : ph + 1;
     if (!grid_barrier(B.bar, tgt, status, [&] {
-          if (!attn && threadIdx.x == 32) gemm_args(P, next, M, pos0, tok, logits, ga);
+          if (!attn && threadIdx.x == 32)
+            gemm_args(P, next, M, cm.rtok, cm.rpos, cm.rslot, logits, ga);
           prefetch_phase(P, ph + 3);
         }))
       return false;
@@ -339,36 +390,60 @@ __device__ bool run_pass(const KParams<W>& P, int M, int pos0, const int* tok, f
 // fixed-point commit (every CTA): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
 // ------------------------------------------------------------------------------------------
 
+// Rows of the next pass: every sentence that is not done contributes its block rows, inputs
+// y_{i-1} then the draft at positions i-1..i+blk-2 (the shift-left of Algorithm 2's appendix
+// note), sentences in order.  All threads of the CTA; misc[0] = the row count.
 template <typename W>
-__device__ __forceinline__ DecState& smem_state() {
-  __shared__ DecState s;
-  return s;
+__device__ void build_rows(const KParams<W>& P, const CommitMem& cm) {
+  const Dims& D = P.D;
+  const int S = P.n_sent;
+  if (threadIdx.x == 0) {
+    int r = 0;
+    for (int s = 0; s < S; ++s) {
+      cm.r0[s] = r;
+      if (!cm.st[s].done) r += cm.st[s].blk;
+    }
+    cm.misc[0] = r;
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int s = warp; s < S; s += kWarps) {
+    const DecState& st = cm.st[s];
+    if (st.done) continue;
+    const int* ys = cm.y + (size_t)s * (D.max_tgt + 1);
+    for (int j = lane; j < st.blk; j += 32) {
+      const int r = cm.r0[s] + j, pos = st.i - 1 + j;
+      cm.rtok[r] = ys[pos];
+      cm.rpos[r] = pos;
+      cm.rsb[r] = s * D.max_tgt;
+      cm.rslot[r] = s * D.max_tgt + pos;
+      cm.rkn[r] = pos + 1;                  // block-causal: keys 0..pos of its own sentence
+      cm.rxb[r] = s * D.max_src;
+      cm.rxn[r] = st.n_src;
+    }
+  }
+  __syncthreads();
 }
 
 // Run after the grid barrier that follows the LM head, by every CTA on its own copy of the
-// state and of y (shared memory): the CTA partials of each row are merged in the same fixed
-// order everywhere, so every CTA takes the same decisions and needs nothing from the others.
-// CTA 0 alone writes the trace to device memory.
+// decoding states and of y (shared memory): the CTA partials of each row are merged in the
+// same fixed order everywhere, so every CTA takes the same decisions and needs nothing from
+// the others.  Thread s decides for sentence s; CTA 0 alone writes the trace (single-sentence
+// decodes).  Ends with the rows of the next pass.
 template <typename W>
 __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
   const SmemLayout SL = smem_layout(D, sizeof(W));
-  int* ntok = reinterpret_cast<int*>(smem + SL.commit);
-  float* nprob = reinterpret_cast<float*>(ntok + D.max_tgt + 1);
-  int* sy = reinterpret_cast<int*>(nprob + D.max_tgt + 1);       // y_0..y_m
-  DecState& ss = smem_state<W>();
-  __shared__ int s_nan, s_scan;
+  const CommitMem cm = commit_mem(D, smem + SL.commit);
   const int tid = threadIdx.x;
   const int lane = tid & 31, warp = tid >> 5;
-  const int blk = ss.blk, i = ss.i, t = ss.n_trace;   // read before thread 0 changes ss
-  if (tid == 0) { s_nan = 0; s_scan = 0; }
-  __syncthreads();
+  const int M = cm.misc[0], S = P.n_sent;
   // per row: the CTA partials merged lane-wise in ascending CTA order (loads issued in
   // batches), then by a fixed butterfly (the merge is symmetric, so every lane ends with the
-  // same result)
+  // same result); a NaN row gets token -1
   constexpr int kBatch = 8;
-  for (int r = warp; r < blk; r += kWarps) {
+  for (int r = warp; r < M; r += kWarps) {
     Partial a{-INFINITY, 0x7fffffff, 0.f, 0};
     for (int c0 = 0; c0 < (int)gridDim.x; c0 += 32 * kBatch) {
       Partial v[kBatch];
@@ -387,39 +462,43 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
       partial_merge(a, b);
     }
     if (lane == 0) {
-      ntok[r] = a.idx;
-      nprob[r] = 1.0f / a.sum;
-      if (a.nan || a.mx == -INFINITY) atomicOr(&s_nan, 1);
+      cm.ntok[r] = (a.nan || a.mx == -INFINITY) ? -1 : a.idx;
+      cm.nprob[r] = 1.0f / a.sum;
     }
   }
   __syncthreads();
-  if (blockIdx.x == 0 && t < D.max_tgt) {
-    for (int r = tid; r < blk; r += blockDim.x) {
-      B.trace_tok[(size_t)t * D.max_tgt + r] = ntok[r];
-      B.trace_prob[(size_t)t * D.max_tgt + r] = nprob[r];
-    }
-  }
-  if (tid == 0) {
-    DecState st = ss;                              // decisions on a register copy
+  for (int s = tid; s < S; s += blockDim.x) {
+    DecState st = cm.st[s];                        // decisions on a register copy
+    if (st.done) continue;
+    const int r0 = cm.r0[s], blk = st.blk, i = st.i;
+    const int* nt = cm.ntok + r0;
+    const int* ys = cm.y + (size_t)s * (D.max_tgt + 1);
+    bool nan = false;
+    for (int r = 0; r < blk; ++r) nan = nan || nt[r] < 0;
     int c = 0;                                     // leading positions equal to the old draft
-    while (c < blk && ntok[c] == sy[i + c]) ++c;
+    while (c < blk && nt[c] == ys[i + c]) ++c;
     const int stop = c == blk;
     int eos_idx = -1;
     for (int r = 0; r < blk; ++r)
-      if (ntok[r] == D.eos) { eos_idx = r; break; }
+      if (nt[r] == D.eos) { eos_idx = r; break; }
     st.k = st.k + 1;
     const int n_it = st.n_iters + 1;
     st.n_iters = n_it;
+    const int t = st.n_trace;
     if (t < D.max_tgt) {
-      if (blockIdx.x == 0) {
+      if (S == 1 && blockIdx.x == 0) {
         pd_trace_step row;
         row.step = n_it; row.block_start = i; row.block_len = blk; row.n_converged = c;
         row.stop = stop; row.eos_idx = eos_idx;
         B.trace[t] = row;
+        for (int r = 0; r < blk; ++r) {
+          B.trace_tok[(size_t)t * D.max_tgt + r] = nt[r];
+          B.trace_prob[(size_t)t * D.max_tgt + r] = cm.nprob[r0 + r];
+        }
       }
       st.n_trace = t + 1;
     }
-    if (s_nan) {
+    if (nan) {
       st.status = PD_ENAN; st.n_y = i - 1; st.done = 1;
     } else {
       // the block is solved: StopC, the pass cap, or (accepted-prefix rule) the first c + 1
@@ -428,7 +507,7 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
         const bool one_pos = st.method == PD_GREEDY || st.ar_tail;
         if (one_pos) {
           const bool eos_ends = st.ar_tail ? true : (st.stop_at_eos != 0);
-          if (eos_ends && ntok[0] == D.eos) { st.n_y = i; st.done = 1; }
+          if (eos_ends && nt[0] == D.eos) { st.n_y = i; st.done = 1; }
         } else if (st.method == PD_HYBRID_GS_JACOBI && eos_idx >= 0) {
           st.n_y = i + eos_idx;                    // through the EOS (Algorithm 3)
           st.done = 1;
@@ -443,7 +522,7 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
           if (ni > st.m_eff) {
             st.done = 1;
             st.n_y = st.m_eff;
-            s_scan = (st.method == PD_JACOBI || st.method == PD_GS_JACOBI) && st.stop_at_eos;
+            st.scan = (st.method == PD_JACOBI || st.method == PD_GS_JACOBI) && st.stop_at_eos;
           } else {
             st.i = ni;
             const int rest = st.m_eff - ni + 1;
@@ -460,37 +539,49 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
         st.done = 1;
       }
     }
-    ss = st;
+    cm.st[s] = st;
   }
   __syncthreads();
-  for (int r = tid; r < blk; r += blockDim.x) sy[i + r] = ntok[r];   // y_{i:i+blk} <- new
+  for (int r = tid; r < M; r += blockDim.x)        // y_{i:i+blk} <- new, every sentence
+    cm.y[(size_t)(cm.rsb[r] / D.max_tgt) * (D.max_tgt + 1) + cm.rpos[r] + 1] = cm.ntok[r];
   __syncthreads();
-  if (s_scan && tid == 0) {                        // the first EOS among y_1..y_m ends y
-    for (int p = 1; p <= ss.m_eff; ++p)
-      if (sy[p] == D.eos) { ss.n_y = p; break; }
+  for (int s = tid; s < S; s += blockDim.x) {      // the first EOS among y_1..y_m ends y
+    DecState& st = cm.st[s];
+    if (!st.scan) continue;
+    const int* ys = cm.y + (size_t)s * (D.max_tgt + 1);
+    for (int p = 1; p <= st.m_eff; ++p)
+      if (ys[p] == D.eos) { st.n_y = p; break; }
+    st.scan = 0;
   }
   __syncthreads();
+  build_rows(P, cm);
 }
 
-// CTA 0, at the end of a decode: tokens and info from its copy of the state; a failure a
-// device-side wait recorded in the status word (PD_ETIMEOUT) takes precedence.
+// CTA 0, at the end of a decode: tokens and info of every sentence from its copies of the
+// states; a failure a device-side wait recorded in the status word (PD_ETIMEOUT) takes
+// precedence.
 template <typename W>
-__device__ void write_outputs(const KParams<W>& P, const unsigned char* smem) {
+__device__ void write_outputs(const KParams<W>& P, unsigned char* smem) {
   const Dims& D = P.D;
   const SmemLayout SL = smem_layout(D, sizeof(W));
-  const int* sy = reinterpret_cast<const int*>(smem + SL.commit) + 2 * (D.max_tgt + 1);
-  const DecState& ss = smem_state<W>();
+  const CommitMem cm = commit_mem(D, smem + SL.commit);
+  const int S = P.n_sent;
   __syncthreads();
-  if (threadIdx.x == 0 && ss.status != 0) atomicCAS(&P.B.st->status, 0, ss.status);
   if (P.out_info == nullptr) return;
-  const int n_y = ss.n_y;
-  for (int p = threadIdx.x; p < n_y; p += blockDim.x) P.out_y[p] = sy[1 + p];
+  for (int s = 0; s < S; ++s) {
+    const int n_y = cm.st[s].n_y;
+    const int* ys = cm.y + (size_t)s * (D.max_tgt + 1);
+    for (int p = threadIdx.x; p < n_y; p += blockDim.x) P.out_y[(size_t)s * P.out_ld + p] = ys[1 + p];
+  }
   if (threadIdx.x == 0) {
     const int g = atomicAdd(&P.B.st->status, 0);
-    P.out_info[0] = n_y;
-    P.out_info[1] = ss.n_iters;
-    P.out_info[2] = g;
-    P.out_info[3] = ss.n_trace;
+    for (int s = 0; s < S; ++s) {
+      const DecState& st = cm.st[s];
+      P.out_info[4 * s + 0] = st.n_y;
+      P.out_info[4 * s + 1] = st.n_iters;
+      P.out_info[4 * s + 2] = g != 0 ? g : st.status;
+      P.out_info[4 * s + 3] = st.n_trace;
+    }
   }
 }
 
@@ -512,36 +603,45 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   for (int i = threadIdx.x; i < kTlN * 8; i += blockDim.x) s_tl[i / 8][i % 8] = 0;
   __syncthreads();
 #endif
+  const SmemLayout SL = smem_layout(D, sizeof(W));
+  const CommitMem cm = commit_mem(D, smem + SL.commit);
 
-  if (P.debug_len > 0) {
-    run_pass<W>(P, P.debug_len, 0, B.dbg_tok, P.logits, tgt, smem);
+  if (P.debug_len > 0) {                  // teacher-forced rows 0..len-1 of the slot-0 sentence
+    for (int m = threadIdx.x; m < P.debug_len; m += blockDim.x) {
+      cm.rtok[m] = B.dbg_tok[m];
+      cm.rpos[m] = m; cm.rslot[m] = m; cm.rsb[m] = 0; cm.rkn[m] = m + 1;
+      cm.rxb[m] = 0; cm.rxn[m] = P.n_src_s[0];
+    }
+    __syncthreads();
+    run_pass<W>(P, P.debug_len, P.logits, tgt, smem);
     return;
   }
 
-  // every CTA: its copy of the state and of y_0..y_m; InitT = all PAD (Section 3.3)
-  const SmemLayout SL = smem_layout(D, sizeof(W));
-  int* sy = reinterpret_cast<int*>(smem + SL.commit) + 2 * (D.max_tgt + 1);
-  DecState& ss = smem_state<W>();
-  for (int p = threadIdx.x; p <= P.init.max_len; p += blockDim.x) sy[p] = p == 0 ? D.bos : D.pad;
-  if (threadIdx.x == 0) {
-    DecState s = P.init;
-    s.b_eff = s.method == PD_GREEDY ? 1 : (s.method == PD_JACOBI ? s.max_len : s.b);
-    s.m_eff = s.method == PD_HYBRID_GS_JACOBI ? s.h : s.max_len;
-    s.i = 1;
-    s.blk = s.b_eff < s.m_eff ? s.b_eff : s.m_eff;
-    s.k = 0; s.ar_tail = 0; s.n_iters = 0; s.done = 0; s.n_y = 0; s.n_trace = 0;
-    s.status = 0;
-    ss = s;
-    if (blockIdx.x == 0) *status = 0;       // nothing reads it before the first barrier wait
+  // every CTA: its copies of the states and of y_0..y_m; InitT = all PAD (Section 3.3)
+  const int S = P.n_sent;
+  for (int s = threadIdx.x; s < S; s += blockDim.x) {
+    DecState st = P.init;
+    st.max_len = P.max_len_s[s];
+    st.h = (P.init.h <= 0 || P.init.h > st.max_len) ? st.max_len : P.init.h;
+    st.n_src = P.n_src_s[s];
+    st.b_eff = st.method == PD_GREEDY ? 1 : (st.method == PD_JACOBI ? st.max_len : st.b);
+    st.m_eff = st.method == PD_HYBRID_GS_JACOBI ? st.h : st.max_len;
+    st.i = 1;
+    st.blk = st.b_eff < st.m_eff ? st.b_eff : st.m_eff;
+    st.k = 0; st.ar_tail = 0; st.n_iters = 0; st.done = 0; st.n_y = 0; st.n_trace = 0;
+    st.status = 0; st.scan = 0;
+    cm.st[s] = st;
   }
+  for (int e = threadIdx.x; e < S * (D.max_tgt + 1); e += blockDim.x)
+    cm.y[e] = e % (D.max_tgt + 1) == 0 ? D.bos : D.pad;
+  if (blockIdx.x == 0 && threadIdx.x == 0) *status = 0;   // read by no one before a wait
   __syncthreads();
+  build_rows(P, cm);
 
   for (;;) {
-    if (ss.done) break;
-    const int M = ss.blk, pos0 = ss.i - 1;
-    // row r's input is the token at position i-1+r: y_{i-1}, then the block's draft
-    // (the shift-left of Algorithm 2's appendix note)
-    if (!run_pass<W>(P, M, pos0, sy + pos0, nullptr, tgt, smem)) break;
+    const int M = cm.misc[0];
+    if (M == 0) break;
+    if (!run_pass<W>(P, M, nullptr, tgt, smem)) break;
     if (!grid_barrier(B.bar, tgt, status)) break;
     commit<W>(P, smem);
   }
@@ -565,6 +665,9 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
   const EmbedTabs<W> T = embed_tabs(P);
   const bool pre = D.pre_ln != 0;
   const int n = P.n_src;
+  const CommitMem cm = commit_mem(D, smem + SL.commit);
+  for (int m = threadIdx.x; m < n; m += blockDim.x) cm.rpos[m] = m;   // source positions
+  __syncthreads();
 
   for (int l = 0; l < D.Le; ++l) {
     const EncLayerW<W>& L = mw.enc[l];
@@ -580,7 +683,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     GemmArgs<W> g{};
     g.M = n; g.N = 3 * D.d; g.K = D.d;
     if (l == 0) {
-      g.emb_tok = P.enc_tok; g.emb_pos0 = 0; g.x_store = B.ra;
+      g.emb_tok = P.enc_tok; g.emb_pos = cm.rpos; g.x_store = B.ra;   // positions 0..n-1
       if (pre) { g.ln_a_g = mw.enc_lne_g; g.ln_a_b = mw.enc_lne_b; g.ln_b_g = L.ln1g; g.ln_b_b = L.ln1b; }
     } else {
       g.x_src = B.ra;
@@ -594,7 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
-    attn_phase<float, W>(D, B.q, B.k, B.v, B.att, n, -1, n, scratch);
+    attn_phase<float, W>(D, B.q, B.k, B.v, B.att, n, nullptr, nullptr, n, scratch);
     if (!grid_barrier(B.bar, tgt, status)) return;
 
     g = GemmArgs<W>{};
@@ -621,15 +724,18 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     gemm_phase<W>(g, T, D, smem);
     if (!grid_barrier(B.bar, tgt, status)) return;
   }
-  // cross-attention keys and values of every decoder layer from the encoder output
+  // cross-attention keys and values of every decoder layer from the encoder output, into the
+  // sentence's slot
+  const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
+  const size_t slot_off = (size_t)P.enc_slot * D.max_src * D.d;
   for (int l = 0; l < D.Ld; ++l) {
     GemmArgs<W> g{};
     g.M = n; g.N = 2 * D.d; g.K = D.d; g.x_src = B.ra;
     g.ln_b_g = pre ? mw.enc_lnf_g : mw.enc[D.Le - 1].ln2g;
     g.ln_b_b = pre ? mw.enc_lnf_b : mw.enc[D.Le - 1].ln2b;
     g.w = mw.dec[l].wkvc; g.bias = mw.dec[l].bkvc; g.epi = EPI_KVCROSS;
-    g.kdst = B.kcross + (size_t)l * D.max_src * D.d;
-    g.vdst = B.vcross + (size_t)l * D.max_src * D.d;
+    g.kdst = B.kcross + l * cross_ld + slot_off;
+    g.vdst = B.vcross + l * cross_ld + slot_off;
     gemm_plan(g, gridDim.x);
     gemm_phase<W>(g, T, D, smem);
   }
@@ -660,8 +766,8 @@ struct pd_ctx {
   pd::Bufs<__nv_bfloat16> bb{};
   int32_t* d_out_y = nullptr;
   int32_t* d_out_info = nullptr;
-  int n_src = 0;
-  bool encoded = false;
+  int n_src_slot[pd::kMaxBatch] = {};        // source length encoded into each cache slot
+  int n_encoded = 0;                          // slots 0..n_encoded-1 hold encoded sentences
   int64_t launches = 0;
   std::string err;
 };
@@ -702,6 +808,7 @@ bool valid_config(const pd_config* c, std::string* why) {
   for (int id : {c->pad_id, c->eos_id, c->bos_id})
     if (id < 0 || id >= c->vocab) return bad("special ids must be in [0, vocab)");
   if (!(c->ln_eps >= 0.f)) return bad("ln_eps");
+  if (c->max_batch < 0 || c->max_batch > pd::kMaxBatch) return bad("max_batch must be in [0, 64]");
   return true;
 }
 
@@ -814,27 +921,28 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
   PD_TRY(dalloc(c, &B.q, R * d)); PD_TRY(dalloc(c, &B.k, R * d)); PD_TRY(dalloc(c, &B.v, R * d));
   PD_TRY(dalloc(c, &B.att, R * d));
   PD_TRY(dalloc(c, &B.ffh, R * (size_t)D.f));
-  PD_TRY(dalloc(c, &B.kself, (size_t)D.Ld * D.max_tgt * d));
-  PD_TRY(dalloc(c, &B.vself, (size_t)D.Ld * D.max_tgt * d));
-  PD_TRY(dalloc(c, &B.kcross, (size_t)D.Ld * D.max_src * d));
-  PD_TRY(dalloc(c, &B.vcross, (size_t)D.Ld * D.max_src * d));
+  const size_t nb = (size_t)D.max_batch;
+  PD_TRY(dalloc(c, &B.kself, (size_t)D.Ld * nb * D.max_tgt * d));
+  PD_TRY(dalloc(c, &B.vself, (size_t)D.Ld * nb * D.max_tgt * d));
+  PD_TRY(dalloc(c, &B.kcross, (size_t)D.Ld * nb * D.max_src * d));
+  PD_TRY(dalloc(c, &B.vcross, (size_t)D.Ld * nb * D.max_src * d));
   PD_TRY(dalloc(c, &B.part, (size_t)c->grid * R));
   PD_TRY(dalloc(c, &B.st, 1));
   PD_TRY(dalloc(c, &B.trace, (size_t)D.max_tgt));
   PD_TRY(dalloc(c, &B.trace_tok, (size_t)D.max_tgt * D.max_tgt));
   PD_TRY(dalloc(c, &B.trace_prob, (size_t)D.max_tgt * D.max_tgt));
   PD_TRY(dalloc(c, &B.bar, 4));
-  PD_TRY(dalloc(c, &B.src, (size_t)D.max_src));
+  PD_TRY(dalloc(c, &B.src, nb * D.max_src));
   PD_TRY(dalloc(c, &B.dbg_tok, (size_t)D.max_tgt));
-  PD_TRY(dalloc(c, &B.pos_tab, R * d));
+  PD_TRY(dalloc(c, &B.pos_tab, (size_t)D.max_keys * d));
   if (!cfg.learned_pos) {
-    pd::sinusoid_kernel<<<c->n_sm, 256, 0, c->stream>>>(B.pos_tab, (int)R, (int)d);
+    pd::sinusoid_kernel<<<c->n_sm, 256, 0, c->stream>>>(B.pos_tab, D.max_keys, (int)d);
     PD_CUDA(c, cudaGetLastError());
     PD_CUDA(c, cudaStreamSynchronize(c->stream));
     c->launches += 1;
   }
-  PD_TRY(dalloc(c, &c->d_out_y, (size_t)D.max_tgt));
-  PD_TRY(dalloc(c, &c->d_out_info, 4));
+  PD_TRY(dalloc(c, &c->d_out_y, nb * D.max_tgt));
+  PD_TRY(dalloc(c, &c->d_out_info, 4 * nb));
   PD_CUDA(c, cudaMemset(B.st, 0, sizeof(pd::DecState)));
   PD_CUDA(c, cudaMemset(B.bar, 0, 4 * sizeof(unsigned)));
 
@@ -857,14 +965,17 @@ pd::KParams<W> base_params(pd_ctx* c) {
   P.D = c->D;
   P.mw = static_cast<const pd::ModelW<W>*>(c->mw_dev);
   P.B = bufs<W>(c);
-  P.n_src = c->n_src;
+  for (int s = 0; s < pd::kMaxBatch; ++s) P.n_src_s[s] = c->n_src_slot[s];
   return P;
 }
 
+// reset_status: clear the status word first (every encode but the later ones of a batch, whose
+// failures must survive until the batch is checked)
 template <typename W>
-pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P) {
+pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P, bool reset_status = true) {
   PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).bar, 0, 4 * sizeof(unsigned), c->stream));
-  if (encode) PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).st, 0, sizeof(pd::DecState), c->stream));
+  if (encode && reset_status)
+    PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).st, 0, sizeof(pd::DecState), c->stream));
   void* args[] = {&P};
   const void* fn = encode ? (const void*)pd::encode_kernel<W> : (const void*)pd::decode_kernel<W>;
   PD_CUDA(c, cudaLaunchCooperativeKernel(fn, dim3(c->grid), dim3(pd::kThreads), args, c->smem,
@@ -874,28 +985,32 @@ pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P) {
 }
 
 template <typename W>
-pd_status encode_impl(pd_ctx* c, const int32_t* d_src, int n) {
+pd_status encode_impl(pd_ctx* c, const int32_t* d_src, int n, int slot, bool reset_status) {
   pd::KParams<W> P = base_params<W>(c);
   P.n_src = n;
+  P.enc_slot = slot;
   P.enc_tok = d_src;
-  PD_TRY(launch<W>(c, true, P));
-  c->n_src = n;
-  c->encoded = true;
+  PD_TRY(launch<W>(c, true, P, reset_status));
+  c->n_src_slot[slot] = n;
   return PD_OK;
 }
 
+// max_len: per-sentence values (host), or nullptr for p->max_len everywhere
 template <typename W>
-pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int32_t* d_y, int32_t* d_info) {
+pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int n_sent, const int32_t* max_len,
+                      int32_t* d_y, int y_ld, int32_t* d_info) {
   pd::KParams<W> P = base_params<W>(c);
   P.init = pd::DecState{};
   P.init.method = p->method;
   P.init.b = p->b;
-  P.init.max_len = p->max_len;
-  P.init.h = (p->h <= 0 || p->h > p->max_len) ? p->max_len : p->h;
+  P.init.h = p->h;
   P.init.stop_at_eos = p->stop_at_eos;
   P.init.max_passes = p->max_passes;
   P.init.stop_rule = p->stop_rule;
+  P.n_sent = n_sent;
+  for (int s = 0; s < n_sent; ++s) P.max_len_s[s] = max_len ? max_len[s] : p->max_len;
   P.out_y = d_y;
+  P.out_ld = y_ld;
   P.out_info = d_info;
   return launch<W>(c, false, P);
 }
@@ -908,19 +1023,29 @@ pd_status debug_impl(pd_ctx* c, int len, float* d_logits) {
   return launch<W>(c, false, P);
 }
 
-pd_status check_params(pd_ctx* c, const pd_decode_params* p) {
+// n_sent sentences (slots 0..n_sent-1), max_len per sentence (nullptr: p->max_len for all)
+pd_status check_params(pd_ctx* c, const pd_decode_params* p, int n_sent = 1,
+                       const int32_t* max_len = nullptr) {
   if (!p) return fail(c, PD_EINVAL, "params is NULL");
   if (p->method < PD_GREEDY || p->method > PD_HYBRID_GS_JACOBI) return fail(c, PD_EINVAL, "method");
-  if (p->max_len < 1 || p->max_len > c->cfg.max_tgt_len)
-    return fail(c, PD_EINVAL, "max_len must be in [1, max_tgt_len]");
   if ((p->method == PD_GS_JACOBI || p->method == PD_HYBRID_GS_JACOBI) && p->b < 1)
     return fail(c, PD_EINVAL, "b must be >= 1");
   if (p->max_passes < 0) return fail(c, PD_EINVAL, "max_passes must be >= 0");
   if (p->stop_rule != PD_STOP_UNCHANGED && p->stop_rule != PD_STOP_PREFIX)
     return fail(c, PD_EINVAL, "stop_rule");
-  if (c->cfg.learned_pos && p->max_len > c->cfg.max_pos)
-    return fail(c, PD_EINVAL, "max_len exceeds the learned position table");
-  if (!c->encoded) return fail(c, PD_ESTATE, "pd_decode before pd_encode");
+  if (n_sent < 1 || n_sent > c->D.max_batch) return fail(c, PD_EINVAL, "n_sent must be in [1, max_batch]");
+  long rows = 0;                                  // rows of the widest pass
+  for (int s = 0; s < n_sent; ++s) {
+    const int m = max_len ? max_len[s] : p->max_len;
+    if (m < 1 || m > c->cfg.max_tgt_len)
+      return fail(c, PD_EINVAL, "max_len must be in [1, max_tgt_len]");
+    if (c->cfg.learned_pos && m > c->cfg.max_pos)
+      return fail(c, PD_EINVAL, "max_len exceeds the learned position table");
+    const int b_eff = p->method == PD_GREEDY ? 1 : (p->method == PD_JACOBI ? m : p->b);
+    rows += b_eff < m ? b_eff : m;
+  }
+  if (rows > c->D.rows) return fail(c, PD_EINVAL, "the sentences' blocks exceed the rows of a pass");
+  if (c->n_encoded < n_sent) return fail(c, PD_ESTATE, "pd_decode before pd_encode");
   return PD_OK;
 }
 
@@ -954,7 +1079,10 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   D.pad = cfg->pad_id; D.eos = cfg->eos_id; D.bos = cfg->bos_id;
   D.eps = cfg->ln_eps; D.emb_scale = sqrtf((float)cfg->d_model);
   D.max_src = cfg->max_src_len; D.max_tgt = cfg->max_tgt_len;
-  D.rows = D.max_src > D.max_tgt ? D.max_src : D.max_tgt;
+  D.max_keys = D.max_src > D.max_tgt ? D.max_src : D.max_tgt;
+  D.max_batch = cfg->max_batch > 1 ? cfg->max_batch : 1;
+  const long batch_rows = std::min<long>((long)D.max_batch * D.max_tgt, pd::kMaxPassRows);
+  D.rows = (int)std::max<long>(D.max_keys, batch_rows);
   c->blob_bytes = nbytes;
   pd_status s = PD_OK;
   cudaError_t e = cudaGetDevice(&c->device);
@@ -1004,8 +1132,11 @@ pd_status pd_encode_device(pd_ctx* c, const int32_t* d_src, int n_src) {
     return fail(c, PD_EINVAL, "n_src must be in [1, max_src_len]");
   if (c->cfg.learned_pos && n_src > c->cfg.max_pos)
     return fail(c, PD_EINVAL, "n_src exceeds the learned position table");
-  return c->cfg.dtype == PD_DTYPE_BF16 ? encode_impl<__nv_bfloat16>(c, d_src, n_src)
-                                       : encode_impl<float>(c, d_src, n_src);
+  c->n_encoded = 0;
+  PD_TRY(c->cfg.dtype == PD_DTYPE_BF16 ? encode_impl<__nv_bfloat16>(c, d_src, n_src, 0, true)
+                                       : encode_impl<float>(c, d_src, n_src, 0, true));
+  c->n_encoded = 1;
+  return PD_OK;
 }
 
 pd_status pd_encode(pd_ctx* c, const int32_t* src, int n_src) {
@@ -1022,7 +1153,57 @@ pd_status pd_encode(pd_ctx* c, const int32_t* src, int n_src) {
   pd::DecState* dst = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.st : c->bf.st;
   PD_CUDA(c, cudaMemcpy(&st, &dst->status, sizeof(int), cudaMemcpyDeviceToHost));
   if (st != 0) {
-    c->encoded = false;
+    c->n_encoded = 0;
+    return fail(c, (pd_status)st, "encoder kernel reported a failure");
+  }
+  return PD_OK;
+}
+
+pd_status pd_encode_batch_device(pd_ctx* c, const int32_t* d_src, const int32_t* offsets,
+                                 int n_sent) {
+  if (!c) return PD_EINVAL;
+  if (!d_src || !offsets || n_sent < 1 || n_sent > c->D.max_batch)
+    return fail(c, PD_EINVAL, "d_src, offsets and n_sent in [1, max_batch] are required");
+  for (int s = 0; s < n_sent; ++s) {
+    const int n = offsets[s + 1] - offsets[s];
+    if (offsets[s] < 0 || n < 1 || n > c->cfg.max_src_len)
+      return fail(c, PD_EINVAL, "every sentence length must be in [1, max_src_len]");
+    if (c->cfg.learned_pos && n > c->cfg.max_pos)
+      return fail(c, PD_EINVAL, "a sentence exceeds the learned position table");
+  }
+  c->n_encoded = 0;
+  for (int s = 0; s < n_sent; ++s) {
+    const int n = offsets[s + 1] - offsets[s];
+    PD_TRY(c->cfg.dtype == PD_DTYPE_BF16
+               ? encode_impl<__nv_bfloat16>(c, d_src + offsets[s], n, s, s == 0)
+               : encode_impl<float>(c, d_src + offsets[s], n, s, s == 0));
+  }
+  c->n_encoded = n_sent;
+  return PD_OK;
+}
+
+pd_status pd_encode_batch(pd_ctx* c, const int32_t* src, const int32_t* offsets, int n_sent) {
+  if (!c) return PD_EINVAL;
+  if (!src || !offsets || n_sent < 1 || n_sent > c->D.max_batch)
+    return fail(c, PD_EINVAL, "src, offsets and n_sent in [1, max_batch] are required");
+  if (offsets[0] != 0) return fail(c, PD_EINVAL, "offsets[0] must be 0");
+  for (int s = 0; s < n_sent; ++s) {
+    const int n = offsets[s + 1] - offsets[s];
+    if (n < 1 || n > c->cfg.max_src_len)
+      return fail(c, PD_EINVAL, "every sentence length must be in [1, max_src_len]");
+  }
+  const int total = offsets[n_sent];
+  for (int k = 0; k < total; ++k)
+    if (src[k] < 0 || src[k] >= c->cfg.vocab) return fail(c, PD_EINVAL, "source id out of range");
+  int32_t* dsrc = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.src : c->bf.src;
+  PD_CUDA(c, cudaMemcpyAsync(dsrc, src, total * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  PD_TRY(pd_encode_batch_device(c, dsrc, offsets, n_sent));
+  PD_CUDA(c, cudaStreamSynchronize(c->stream));
+  int st = 0;
+  pd::DecState* dst = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.st : c->bf.st;
+  PD_CUDA(c, cudaMemcpy(&st, &dst->status, sizeof(int), cudaMemcpyDeviceToHost));
+  if (st != 0) {
+    c->n_encoded = 0;
     return fail(c, (pd_status)st, "encoder kernel reported a failure");
   }
   return PD_OK;
@@ -1032,8 +1213,49 @@ pd_status pd_decode_device(pd_ctx* c, const pd_decode_params* p, int32_t* d_y, i
   if (!c) return PD_EINVAL;
   PD_TRY(check_params(c, p));
   if (!d_y || !d_info) return fail(c, PD_EINVAL, "d_y and d_info are required");
-  return c->cfg.dtype == PD_DTYPE_BF16 ? decode_impl<__nv_bfloat16>(c, p, d_y, d_info)
-                                       : decode_impl<float>(c, p, d_y, d_info);
+  return c->cfg.dtype == PD_DTYPE_BF16
+             ? decode_impl<__nv_bfloat16>(c, p, 1, nullptr, d_y, p->max_len, d_info)
+             : decode_impl<float>(c, p, 1, nullptr, d_y, p->max_len, d_info);
+}
+
+pd_status pd_decode_batch_device(pd_ctx* c, const pd_decode_params* p, int n_sent,
+                                 const int32_t* max_len, int32_t* d_y, int y_ld, int32_t* d_info) {
+  if (!c) return PD_EINVAL;
+  PD_TRY(check_params(c, p, n_sent, max_len));
+  if (!d_y || !d_info) return fail(c, PD_EINVAL, "d_y and d_info are required");
+  for (int s = 0; s < n_sent; ++s)
+    if ((max_len ? max_len[s] : p->max_len) > y_ld) return fail(c, PD_EINVAL, "y_ld < max_len");
+  return c->cfg.dtype == PD_DTYPE_BF16
+             ? decode_impl<__nv_bfloat16>(c, p, n_sent, max_len, d_y, y_ld, d_info)
+             : decode_impl<float>(c, p, n_sent, max_len, d_y, y_ld, d_info);
+}
+
+pd_status pd_decode_batch(pd_ctx* c, const pd_decode_params* p, int n_sent,
+                          const int32_t* max_len, int32_t* y, int y_ld, int32_t* n_y,
+                          int32_t* n_iters) {
+  if (!c) return PD_EINVAL;
+  if (!y || !n_y || !n_iters) return fail(c, PD_EINVAL, "y, n_y and n_iters are required");
+  const int ld = c->cfg.max_tgt_len;
+  PD_TRY(pd_decode_batch_device(c, p, n_sent, max_len, c->d_out_y, ld, c->d_out_info));
+  std::vector<int32_t> info(4 * (size_t)n_sent);
+  PD_CUDA(c, cudaMemcpyAsync(info.data(), c->d_out_info, info.size() * sizeof(int32_t),
+                             cudaMemcpyDeviceToHost, c->stream));
+  PD_CUDA(c, cudaStreamSynchronize(c->stream));
+  const int w = std::min(y_ld, ld);
+  PD_CUDA(c, cudaMemcpy2D(y, y_ld * sizeof(int32_t), c->d_out_y, ld * sizeof(int32_t),
+                          w * sizeof(int32_t), n_sent, cudaMemcpyDeviceToHost));
+  int first_bad = 0;
+  for (int s = 0; s < n_sent; ++s) {
+    const int m = max_len ? max_len[s] : p->max_len;
+    n_y[s] = info[4 * s] < 0 ? 0 : std::min(info[4 * s], m);
+    n_iters[s] = info[4 * s + 1];
+    if (!first_bad && info[4 * s + 2] != 0) first_bad = info[4 * s + 2];
+  }
+  if (first_bad != 0)
+    return fail(c, (pd_status)first_bad, first_bad == PD_ENOTCONV ? "pass budget exhausted"
+                                         : first_bad == PD_ENAN ? "NaN in the logits"
+                                         : "decode kernel reported a failure");
+  return PD_OK;
 }
 
 pd_status pd_decode(pd_ctx* c, const pd_decode_params* p, int32_t* y, int* n_y, int* n_iters,
@@ -1087,7 +1309,7 @@ pd_status pd_debug_logits(pd_ctx* c, const int32_t* y_in, int len, float* logits
   if (c->cfg.learned_pos && len > c->cfg.max_pos) return fail(c, PD_EINVAL, "len exceeds max_pos");
   for (int k = 0; k < len; ++k)
     if (y_in[k] < 0 || y_in[k] >= c->cfg.vocab) return fail(c, PD_EINVAL, "token id out of range");
-  if (!c->encoded) return fail(c, PD_ESTATE, "pd_debug_logits before pd_encode");
+  if (c->n_encoded < 1) return fail(c, PD_ESTATE, "pd_debug_logits before pd_encode");
   int* dtok = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.dbg_tok : c->bf.dbg_tok;
   PD_CUDA(c, cudaMemcpyAsync(dtok, y_in, len * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
   float* dl = nullptr;
@@ -1165,7 +1387,7 @@ pd_status pd_debug_logits_static(pd_ctx* c, const int32_t* y_in, int len, float*
   if (c->cfg.learned_pos && len > c->cfg.max_pos) return fail(c, PD_EINVAL, "len exceeds max_pos");
   for (int k = 0; k < len; ++k)
     if (y_in[k] < 0 || y_in[k] >= c->cfg.vocab) return fail(c, PD_EINVAL, "token id out of range");
-  if (!c->encoded) return fail(c, PD_ESTATE, "pd_debug_logits_static before pd_encode");
+  if (c->n_encoded < 1) return fail(c, PD_ESTATE, "pd_debug_logits_static before pd_encode");
   float* dl = nullptr;
   PD_TRY(static_logits_addr(c, &dl));
   int* dtok = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.dbg_tok : c->bf.dbg_tok;

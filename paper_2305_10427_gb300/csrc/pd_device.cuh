@@ -25,6 +25,8 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kMTile = 8;           // rows per GEMM tile
 constexpr int kNCol = 4;            // output columns per warp iteration (kNCol * kMTile == 32)
 constexpr int kMaxLayers = 16;
+constexpr int kMaxBatch = 64;        // sentences of one batched decode
+constexpr int kMaxPassRows = 512;    // rows of one batched decoder pass
 constexpr unsigned long long kWaitNs = 10000000000ull;  // bounded device waits: 10 s
 
 enum Epi : int {
@@ -61,7 +63,10 @@ struct Dims {
   int act, pre_ln, learned_pos, max_pos;
   int pad, eos, bos;
   float eps, emb_scale;
-  int max_src, max_tgt, rows;   // rows = max(max_src, max_tgt): activation buffer rows
+  int max_src, max_tgt;
+  int max_keys;    // max(max_src, max_tgt): rows of the position table, keys of an attention row
+  int max_batch;   // sentences one decode carries (cache slots per layer)
+  int rows;        // activation rows: max(max_keys, min(max_batch * max_tgt, kMaxPassRows))
 };
 
 // Per-CTA partial of the LM-head argmax for one row.
@@ -81,6 +86,8 @@ struct DecState {
   int i, blk, k;          // block start (1-based), block length, passes in this block
   int ar_tail;            // hybrid: past h, one position per pass
   int n_iters, done, status, n_y, n_trace;
+  int n_src;              // source length of the sentence (cross-attention keys)
+  int scan;               // the first EOS of y_1..y_m is still to be found
 };
 
 template <typename W>
@@ -90,8 +97,8 @@ struct Bufs {
   float *q, *k, *v;            // [rows][d]
   W* att;                      // [rows][d] attention output, rounded to W (the O input type)
   W* ffh;                      // [rows][f] FFN hidden, rounded to W (FFN2's input type)
-  W *kself, *vself;            // [Ld][max_tgt][d]
-  W *kcross, *vcross;          // [Ld][max_src][d]
+  W *kself, *vself;            // [Ld][max_batch * max_tgt][d]: sentence s at slots s * max_tgt..
+  W *kcross, *vcross;          // [Ld][max_batch * max_src][d]: sentence s at rows s * max_src..
   Partial* part;               // [grid][rows]
   DecState* st;
   pd_trace_step* trace;        // [max_tgt]
@@ -298,7 +305,7 @@ struct GemmArgs {
   const float* x_src;
   const W* xw_src;          // input rows already rounded to W (plain copy; instead of x_src)
   const int* emb_tok;
-  int emb_pos0;
+  const int* emb_pos;       // per-row positions of the embedded rows
   const W *ln_a_g, *ln_a_b;
   float* x_store;
   const W *ln_b_g, *ln_b_b;
@@ -309,9 +316,9 @@ struct GemmArgs {
   W* out_w;                 // [M][ld] for ACT
   int ld;
   const float* resid;       // [M][ld]
-  W *kdst, *vdst;           // QKV: cache rows (slot = slot0 + m); KVCROSS: cross caches
+  W *kdst, *vdst;           // QKV: cache rows slot[m]; KVCROSS: cross caches
   float *kdst_f, *vdst_f;   // QKV into fp32 buffers (encoder)
-  int slot0;
+  const int* slot;          // QKV into kdst / vdst: per-row cache slots
   Partial* part;            // ARGMAX: [grid][rows_ld]
   int part_ld;
   // How the phase is divided over the grid (gemm_plan): column groups, K-steps per warp,
@@ -544,7 +551,7 @@ __device__ void stage_x(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims&
     if (g.emb_tok != nullptr) {
       int t = g.emb_tok[m];
       t = t < 0 ? 0 : (t >= D.V ? D.V - 1 : t);
-      const int p = g.emb_pos0 + m;
+      const int p = g.emb_pos[m];
       const W* er = T.E + (size_t)t * K;
 #pragma unroll
       for (int i = 0; i < kMaxRowRegs; ++i) {
@@ -705,7 +712,7 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
             g.out[(size_t)m * D.d + cc] = v;
           } else if (g.kdst != nullptr) {
             W* dst = which == 1 ? g.kdst : g.vdst;
-            dst[(size_t)(g.slot0 + m) * D.d + cc] = from_f<W>(v);
+            dst[(size_t)g.slot[m] * D.d + cc] = from_f<W>(v);
           } else {
             float* dst = which == 1 ? g.kdst_f : g.vdst_f;
             dst[(size_t)m * D.d + cc] = v;
@@ -800,26 +807,30 @@ __device__ __forceinline__ void add_pv32(const float* v, float p, float (&acc)[3
 // One warp per (row m, head): lane l owns keys l, l+32, ...  Scores, softmax and the
 // p-weighted value sums are accumulated per lane in ascending key order, then combined by
 // fixed butterflies, so a row's result depends only on its own query and keys.
-// causal_pos0 >= 0: row m attends keys 0..causal_pos0+m; else all n_keys keys.
+// Row m attends the rkeys[m] keys starting at key row rbase[m] of kc / vc (its sentence's
+// cache: causal rows pass their position + 1); without the arrays every row attends the first
+// n_keys keys.
 template <typename KV, typename O>
 __device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV* kc, const KV* vc,
-                           O* out, int M, int causal_pos0, int n_keys, float* scratch) {
+                           O* out, int M, const int* rbase, const int* rkeys, int n_keys,
+                           float* scratch) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int gw = warp * gridDim.x + blockIdx.x;     // items dealt to CTAs round robin
   const int tw = gridDim.x * kWarps;
   const int dh = D.dh;
-  float* qs = scratch + (size_t)warp * (128 + D.rows + 4);
+  float* qs = scratch + (size_t)warp * (128 + D.max_keys + 4);
   float* ps = qs + 128;
   const float scale = 1.0f / sqrtf((float)dh);
   for (int it = gw; it < M * D.H; it += tw) {
     const int m = it / D.H, h = it - m * D.H;
-    const int T = causal_pos0 >= 0 ? causal_pos0 + m + 1 : n_keys;
+    const int T = rkeys != nullptr ? rkeys[m] : n_keys;
+    const size_t kb = rbase != nullptr ? (size_t)rbase[m] * D.d : 0;
     for (int e = lane; e < dh; e += 32) qs[e] = q[(size_t)m * D.d + h * dh + e] * scale;
     __syncwarp();
     float lmax = -INFINITY;
     for (int j = lane; j < T; j += 32) {
-      const float s = key_dot<KV>(kc + (size_t)j * D.d + h * dh, qs, dh);
+      const float s = key_dot<KV>(kc + kb + (size_t)j * D.d + h * dh, qs, dh);
       ps[j] = s;
       lmax = fmaxf(lmax, s);
     }
@@ -837,7 +848,7 @@ __device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV*
       for (int e = 0; e < 32; ++e) acc[e] = 0.f;
       for (int j = lane; j < T; j += 32) {
         const float p = ps[j];
-        add_pv32(vc + (size_t)j * D.d + h * dh + c0, p, acc);
+        add_pv32(vc + kb + (size_t)j * D.d + h * dh + c0, p, acc);
       }
       const float tot = reduce_scatter32(acc);
       out[(size_t)m * D.d + h * dh + c0 + lane] = from_f<O>(tot / sum);

@@ -49,7 +49,7 @@ def test_invalid_configs_are_rejected_before_cuda(lib):
     import dataclasses
     for bad in (dict(d_model=200), dict(n_heads=3), dict(d_ff=100), dict(n_dec_layers=0),
                 dict(n_enc_layers=17), dict(dtype=5), dict(eos_id=9000), dict(max_tgt_len=0),
-                dict(n_heads=1)):
+                dict(n_heads=1), dict(max_batch=65), dict(max_batch=-1)):
         cfg = dataclasses.replace(good, **bad)
         assert pkg.weights_nbytes(cfg) == 0, bad
         c = cfg._c()
@@ -74,6 +74,10 @@ def test_null_context_calls(lib):
     assert lib.pd_encode(None, None, 3) == B.PD_EINVAL
     assert lib.pd_decode_device(None, None, None, None) == B.PD_EINVAL
     assert lib.pd_debug_wait_timeout(None, 1000, None) == B.PD_EINVAL
+    assert lib.pd_encode_batch(None, None, None, 1) == B.PD_EINVAL
+    assert lib.pd_encode_batch_device(None, None, None, 1) == B.PD_EINVAL
+    assert lib.pd_decode_batch(None, None, 1, None, None, 0, None, None) == B.PD_EINVAL
+    assert lib.pd_decode_batch_device(None, None, 1, None, None, 0, None) == B.PD_EINVAL
     assert lib.pd_launch_count(None) == 0
     assert lib.pd_last_error(None) == b"context is NULL"
     lib.pd_destroy(None)
