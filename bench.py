@@ -35,7 +35,7 @@ METRIC = "translated tokens/s at batch 1, GS-Jacobi vs greedy AR; HBM GB/s % of 
 FALLBACK_HBM_GBS = 6800.0
 
 # DRAM bytes (read + write) per decoder pass of decode_kernel<bf16> on this workload, from one
-# ncu capture (profiles/decode_kernel_marian_bf16.md), valid only for the kernel code whose
+# ncu capture of this workload, valid only for the kernel code whose
 # SHA-256 (comments and blank lines left out) is recorded here; other code reports traffic null.
 DRAM_BYTES_PER_PASS = 15.11e6
 DRAM_SOURCES_SHA256 = "2db46da6b4bb25f97141953e928ff441beb2fa65a92e178743d42c3a07d682a1"

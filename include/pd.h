@@ -187,7 +187,8 @@ pd_status pd_decode_batch_device(pd_ctx* ctx, const pd_decode_params* p, int n_s
 /* Test-only: teacher-forced logits of one decoder pass over the input tokens y_in[0..len)
  * at positions 0..len-1 (row t scores position t+1, Eq. 1) for the sentence last encoded.
  * logits: host float32 [len][vocab].  Allocates a temporary device buffer; overwrites the
- * decoder's key/value cache. */
+ * decoder's key/value cache.  Synchronous; PD_ETIMEOUT if a device wait gave up during the
+ * pass (no logits are returned then). */
 pd_status pd_debug_logits(pd_ctx* ctx, const int32_t* y_in, int len, float* logits);
 
 /* Test-only, allocation-free variant of pd_debug_logits (the paper has no counterpart: this
@@ -196,11 +197,12 @@ pd_status pd_debug_logits(pd_ctx* ctx, const int32_t* y_in, int len, float* logi
  * results as pd_debug_logits, but the logits are staged in a fixed 4 MiB array inside the
  * library's device image instead of a per-call allocation, so len * vocab must not exceed
  * 1,048,576 (PD_EINVAL otherwise).  Every GPU that loads the library holds the array until the
- * process exits.  The first call for a device looks up the array's device address (with that
- * device made current for the lookup); make that first call before any stream capture.  All
- * calls share the one array, which keeps the last call's contents: calls that overlap on the
- * GPU (several contexts or threads at once) race and must be serialised by the caller.
- * Synchronous; calls no device allocator. */
+ * process exits.  pd_create looks up the array's device address for its device (current while
+ * it runs) and keeps it in the context, so this call does no set-up of its own.  All calls
+ * share the one array, which keeps the last call's contents: calls that overlap on the GPU
+ * (several contexts or threads at once) race and must be serialised by the caller.  Like
+ * pd_debug_logits it overwrites the decoder's key/value cache and synchronises the context
+ * stream; PD_ETIMEOUT if a device wait gave up during the pass.  Calls no device allocator. */
 pd_status pd_debug_logits_static(pd_ctx* ctx, const int32_t* y_in, int len, float* logits);
 
 /* Test-only failure-detection check (the paper has no counterpart).  Runs, on the context's
@@ -218,7 +220,9 @@ void* pd_stream(pd_ctx* ctx);
 /* Number of the library's kernel launches issued on this context so far. */
 int64_t pd_launch_count(const pd_ctx* ctx);
 
-/* One-line reason for the last failure on ctx ("" if none); valid until the next call. */
+/* One-line reason for the last failure on ctx ("" if none); valid until the next call.  With
+ * ctx = NULL: the reason of the calling thread's last failed pd_create (which returns no
+ * context to ask). */
 const char* pd_last_error(const pd_ctx* ctx);
 
 /* Free every device buffer and the context (NULL is a no-op). */

@@ -184,7 +184,7 @@ class Decoder:
                                  blob.nbytes, ctypes.c_void_p(stream) if stream else None,
                                  ctypes.byref(h))
         if st != PD_OK:
-            raise PdError(st, "pd_create failed (check the configuration and blob size)")
+            raise PdError(st, "pd_create: " + self._lib.pd_last_error(None).decode())
         self._h = h
         self.blob_nbytes = blob.nbytes
 

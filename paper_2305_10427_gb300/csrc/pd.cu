@@ -598,11 +598,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   int* status = &B.st->status;
   load_smem_mw(P);
   load_smem_vectors<W>(D, smem);
-#ifdef PD_TIMELINE
-  if (threadIdx.x == 0) { s_tl_n = 0; s_tl_first = g_tl_first; }
-  for (int i = threadIdx.x; i < kTlN * 8; i += blockDim.x) s_tl[i / 8][i % 8] = 0;
-  __syncthreads();
-#endif
   const SmemLayout SL = smem_layout(D, sizeof(W));
   const CommitMem cm = commit_mem(D, smem + SL.commit);
 
@@ -645,9 +640,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
     if (!grid_barrier(B.bar, tgt, status)) break;
     commit<W>(P, smem);
   }
-#ifdef PD_TIMELINE
-  tl_dump();
-#endif
   if (blockIdx.x == 0) write_outputs(P, smem);
 }
 
@@ -769,6 +761,7 @@ struct pd_ctx {
   int n_src_slot[pd::kMaxBatch] = {};        // source length encoded into each cache slot
   int n_encoded = 0;                          // slots 0..n_encoded-1 hold encoded sentences
   int64_t launches = 0;
+  float* static_logits = nullptr;              // device address of the fixed logits array
   std::string err;
 };
 
@@ -1015,12 +1008,26 @@ pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int n_sent, const in
   return launch<W>(c, false, P);
 }
 
+// A teacher-forced pass starts with a clear status word, so that a wait that gives up during
+// it (PD_ETIMEOUT) is the only status the caller can read back afterwards (debug_status).
 template <typename W>
 pd_status debug_impl(pd_ctx* c, int len, float* d_logits) {
   pd::KParams<W> P = base_params<W>(c);
   P.debug_len = len;
   P.logits = d_logits;
+  PD_CUDA(c, cudaMemsetAsync(&bufs<W>(c).st->status, 0, sizeof(int), c->stream));
   return launch<W>(c, false, P);
+}
+
+// After the stream has been synchronised: the status a teacher-forced pass left (0 if it ran
+// to the end).
+pd_status debug_status(pd_ctx* c) {
+  int st = 0;
+  const pd::DecState* dst = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.st : c->bf.st;
+  PD_CUDA(c, cudaMemcpy(&st, &dst->status, sizeof(int), cudaMemcpyDeviceToHost));
+  if (st != 0) return fail(c, (pd_status)st, "the teacher-forced pass stopped early (a device "
+                                             "wait gave up); no logits were returned");
+  return PD_OK;
 }
 
 // n_sent sentences (slots 0..n_sent-1), max_len per sentence (nullptr: p->max_len for all)
@@ -1055,6 +1062,11 @@ pd_status check_params(pd_ctx* c, const pd_decode_params* p, int n_sent = 1,
 // C ABI
 // ============================================================================================
 
+static pd_status static_logits_lookup(pd_ctx* c);
+
+// Reason of this thread's last failed pd_create (read through pd_last_error(NULL)).
+static thread_local std::string g_create_err;
+
 extern "C" {
 
 size_t pd_weights_nbytes(const pd_config* cfg) {
@@ -1064,11 +1076,17 @@ size_t pd_weights_nbytes(const pd_config* cfg) {
 
 pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, void* stream,
                     pd_ctx** out) {
-  if (!out) return PD_EINVAL;
+  g_create_err.clear();
+  if (!out) { g_create_err = "out is NULL"; return PD_EINVAL; }
   *out = nullptr;
   std::string why;
-  if (!valid_config(cfg, &why)) return PD_EINVAL;
-  if (!weights || nbytes != pd_weights_nbytes(cfg)) return PD_EINVAL;
+  if (!valid_config(cfg, &why)) { g_create_err = "invalid config: " + why; return PD_EINVAL; }
+  if (!weights) { g_create_err = "weights is NULL"; return PD_EINVAL; }
+  if (nbytes != pd_weights_nbytes(cfg)) {
+    g_create_err = "nbytes is " + std::to_string(nbytes) + ", the blob of this config has " +
+                   std::to_string(pd_weights_nbytes(cfg));
+    return PD_EINVAL;
+  }
   pd_ctx* c = new pd_ctx();
   c->cfg = *cfg;
   Dims& D = c->D;
@@ -1090,6 +1108,8 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   int coop = 0;
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, c->device);
   if (e != cudaSuccess || !coop) {
+    g_create_err = e != cudaSuccess ? std::string("device query: ") + cudaGetErrorString(e)
+                                    : "the device has no cooperative launch";
     pd_destroy(c);
     return PD_ECUDA;
   }
@@ -1098,6 +1118,7 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
     c->stream = static_cast<cudaStream_t>(stream);
   } else {
     if (cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking) != cudaSuccess) {
+      g_create_err = "cudaStreamCreateWithFlags failed";
       pd_destroy(c);
       return PD_ECUDA;
     }
@@ -1105,7 +1126,9 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   }
   s = cfg->dtype == PD_DTYPE_BF16 ? create_impl<__nv_bfloat16>(c, weights)
                                   : create_impl<float>(c, weights);
+  if (s == PD_OK) s = static_logits_lookup(c);
   if (s != PD_OK) {
+    g_create_err = c->err;
     pd_destroy(c);
     return s;
   }
@@ -1318,6 +1341,7 @@ pd_status pd_debug_logits(pd_ctx* c, const int32_t* y_in, int len, float* logits
   pd_status s = c->cfg.dtype == PD_DTYPE_BF16 ? debug_impl<__nv_bfloat16>(c, len, dl)
                                                : debug_impl<float>(c, len, dl);
   cudaError_t e = s == PD_OK ? cudaStreamSynchronize(c->stream) : cudaSuccess;
+  if (s == PD_OK && e == cudaSuccess) s = debug_status(c);
   if (s == PD_OK && e == cudaSuccess) e = cudaMemcpy(logits, dl, nb, cudaMemcpyDeviceToHost);
   cudaFree(dl);
   if (s != PD_OK) return s;
@@ -1340,41 +1364,25 @@ pd_status pd_debug_logits(pd_ctx* c, const int32_t* y_in, int len, float* logits
 namespace {
 
 constexpr size_t kStaticLogitsFloats = (size_t)1 << 20;   // 4 MiB: len * vocab <= 1,048,576
-constexpr int kMaxDevices = 64;
-
-std::mutex g_static_mu;
-float* g_static_dev[kMaxDevices] = {};   // device address of the array, per device
 
 }  // namespace
 
 // In host code this name stands for the array; its device address comes from
-// cudaGetSymbolAddress (done once per device in static_logits_addr).
+// cudaGetSymbolAddress, looked up by static_logits_lookup when a context is created.
 static __device__ __align__(256) float g_static_logits[kStaticLogitsFloats];
 
-namespace {
-
-// Device address of g_static_logits on the context's device, looked up on the first call
-// made for that device (with that device current) and cached.
-pd_status static_logits_addr(pd_ctx* c, float** out) {
-  if (c->device < 0 || c->device >= kMaxDevices) return fail(c, PD_EINVAL, "device index too large");
-  std::lock_guard<std::mutex> lock(g_static_mu);
-  if (g_static_dev[c->device] == nullptr) {
-    int prev = -1;
-    PD_CUDA(c, cudaGetDevice(&prev));
-    if (prev != c->device) PD_CUDA(c, cudaSetDevice(c->device));
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_logits);
-    if (prev != c->device) cudaSetDevice(prev);
-    if (e != cudaSuccess || p == nullptr)
-      return fail(c, PD_ECUDA, std::string("cudaGetSymbolAddress(g_static_logits): ") +
-                                   cudaGetErrorString(e));
-    g_static_dev[c->device] = static_cast<float*>(p);
-  }
-  *out = g_static_dev[c->device];
+// Device address of g_static_logits on the context's device (current while pd_create runs),
+// kept in the context: a context never outlives its device's primary context, so the address
+// stays valid for every later call on it.
+static pd_status static_logits_lookup(pd_ctx* c) {
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_static_logits);
+  if (e != cudaSuccess || p == nullptr)
+    return fail(c, PD_ECUDA, std::string("cudaGetSymbolAddress(g_static_logits): ") +
+                                 cudaGetErrorString(e));
+  c->static_logits = static_cast<float*>(p);
   return PD_OK;
 }
-
-}  // namespace
 
 extern "C" {
 
@@ -1388,13 +1396,14 @@ pd_status pd_debug_logits_static(pd_ctx* c, const int32_t* y_in, int len, float*
   for (int k = 0; k < len; ++k)
     if (y_in[k] < 0 || y_in[k] >= c->cfg.vocab) return fail(c, PD_EINVAL, "token id out of range");
   if (c->n_encoded < 1) return fail(c, PD_ESTATE, "pd_debug_logits_static before pd_encode");
-  float* dl = nullptr;
-  PD_TRY(static_logits_addr(c, &dl));
+  float* dl = c->static_logits;
   int* dtok = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.dbg_tok : c->bf.dbg_tok;
   PD_CUDA(c, cudaMemcpyAsync(dtok, y_in, len * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
   // every element of the [len][vocab] region is written by the kernel: nothing to clear
   PD_TRY(c->cfg.dtype == PD_DTYPE_BF16 ? debug_impl<__nv_bfloat16>(c, len, dl)
                                        : debug_impl<float>(c, len, dl));
+  PD_CUDA(c, cudaStreamSynchronize(c->stream));
+  PD_TRY(debug_status(c));
   PD_CUDA(c, cudaMemcpyAsync(logits, dl, (size_t)len * c->cfg.vocab * sizeof(float),
                              cudaMemcpyDeviceToHost, c->stream));
   PD_CUDA(c, cudaStreamSynchronize(c->stream));
@@ -1428,18 +1437,10 @@ pd_status pd_debug_wait_timeout(pd_ctx* c, uint64_t limit_ns, int* status) {
 
 void* pd_stream(pd_ctx* c) { return c ? (void*)c->stream : nullptr; }
 
-#ifdef PD_TIMELINE
-// Development builds only: record the per-CTA timeline of barrier intervals first..first+51.
-int pd_debug_set_tl(void* dptr, int first) {
-  if (cudaMemcpyToSymbol(pd::g_tl, &dptr, sizeof(dptr)) != cudaSuccess) return -3;
-  if (cudaMemcpyToSymbol(pd::g_tl_first, &first, sizeof(first)) != cudaSuccess) return -3;
-  return 0;
-}
-#endif
 
 int64_t pd_launch_count(const pd_ctx* c) { return c ? c->launches : 0; }
 
-const char* pd_last_error(const pd_ctx* c) { return c ? c->err.c_str() : "context is NULL"; }
+const char* pd_last_error(const pd_ctx* c) { return c ? c->err.c_str() : g_create_err.c_str(); }
 
 void pd_destroy(pd_ctx* c) {
   if (!c) return;

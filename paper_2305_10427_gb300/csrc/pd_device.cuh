@@ -174,41 +174,6 @@ __device__ __forceinline__ float act_fn(float v, int act) {
 // grid barriers with bounded waits
 // ------------------------------------------------------------------------------------------
 
-#ifdef PD_TIMELINE
-// Development-only timeline: per-CTA clock marks of kTlN consecutive barrier intervals (from
-// interval g_tl_first on), held in shared memory while the kernel runs and written out at its
-// end.  Marks of an interval: 0 / 4 release of the barrier that opens it (clock64 /
-// globaltimer), 6 GEMM tile start, 7 this warp's rows staged, 1 all rows staged, 2 tile
-// products and epilogue done, 3 / 5 arrival at the barrier that closes it.
-constexpr int kTlN = 52;
-__device__ unsigned long long* g_tl = nullptr;   // [kTlN][grid][8]
-__device__ int g_tl_first = 0;
-__shared__ int s_tl_n, s_tl_first;
-__shared__ unsigned long long s_tl[kTlN][8];
-__device__ __forceinline__ void tl_mark(int k, bool gt) {
-  if (threadIdx.x == 0) {
-    const int i = s_tl_n - s_tl_first;
-    if ((unsigned)i < (unsigned)kTlN) {
-      unsigned long long v;
-      if (gt) { asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(v)); }
-      else { v = clock64(); }
-      s_tl[i][k] = v;
-    }
-  }
-}
-__device__ __forceinline__ void tl_dump() {
-  if (threadIdx.x == 0 && g_tl != nullptr)
-    for (int i = 0; i < kTlN; ++i)
-      for (int k = 0; k < 8; ++k) g_tl[((size_t)i * gridDim.x + blockIdx.x) * 8 + k] = s_tl[i][k];
-}
-#define TL(k) tl_mark(k, false)
-#define TLG(k) tl_mark(k, true)
-#define TL_NEXT() do { if (threadIdx.x == 0) ++s_tl_n; } while (0)
-#else
-#define TL(k) do { } while (0)
-#define TLG(k) do { } while (0)
-#define TL_NEXT() do { } while (0)
-#endif
 
 
 __device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
@@ -255,7 +220,6 @@ __device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, in
   __shared__ int s_ok;
   __syncthreads();
   target += gridDim.x;
-  TL(3); TLG(5);
   if (threadIdx.x == 0) {
     red_release_add(bar, 1u);
   }
@@ -263,7 +227,6 @@ __device__ __forceinline__ bool grid_barrier(unsigned* bar, unsigned& target, in
   if (threadIdx.x == 0) {
     s_ok = spin_until(bar, bar, target, status);
   }
-  TL_NEXT(); TL(0); TLG(4);
   __syncthreads();
   return s_ok != 0;
 }
@@ -676,12 +639,9 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
   const int c = lane / kMTile, r = lane % kMTile;   // the (column, row) this lane finishes
   for (int m0 = 0; m0 < g.M; m0 += kMTile) {
     const int mt = g.M - m0 < kMTile ? g.M - m0 : kMTile;
-    if (m0 == 0) TL(6);
     __syncthreads();
     stage_x(g, T, D, m0, mt, xs);
-    if (m0 == 0) TL(7);
     __syncthreads();
-    if (m0 == 0) TL(1);
     float amx = -INFINITY, asum = 0.f;
     int aidx = 0x7fffffff, anan = 0;
     for (int base = 0; base < ngroups; base += stride) {
@@ -729,7 +689,6 @@ __device__ __noinline__ void gemm_phase(const GemmArgs<W>& g, const EmbedTabs<W>
         case EPI_LOGITS: g.out[(size_t)m * g.ld + n] = v; break;
       }
     }
-    if (m0 == 0) TL(2);
     if (g.epi == EPI_ARGMAX) {
       // lane c*kMTile + r of a part-0 warp holds row r over its columns n0 + c.  Row r's
       // kWarps * kNCol partials are merged by warp r: lane l takes entries l, l + 32, ...

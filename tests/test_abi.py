@@ -79,8 +79,22 @@ def test_null_context_calls(lib):
     assert lib.pd_decode_batch(None, None, 1, None, None, 0, None, None) == B.PD_EINVAL
     assert lib.pd_decode_batch_device(None, None, 1, None, None, 0, None) == B.PD_EINVAL
     assert lib.pd_launch_count(None) == 0
-    assert lib.pd_last_error(None) == b"context is NULL"
     lib.pd_destroy(None)
+
+
+def test_create_failure_reason(lib):
+    """pd_create keeps the reason of its failure for pd_last_error(NULL)."""
+    cfg = pkg.Config.from_spec(synth.TINY, 64, 128)
+    c = cfg._c()
+    h = ctypes.c_void_p()
+    blob = np.zeros(10, dtype=np.float32)
+    assert lib.pd_create(ctypes.byref(c), blob.ctypes.data_as(ctypes.c_void_p), blob.nbytes,
+                         None, ctypes.byref(h)) == B.PD_EINVAL
+    assert b"nbytes is 40" in lib.pd_last_error(None)
+    c.d_model = 100
+    assert lib.pd_create(ctypes.byref(c), blob.ctypes.data_as(ctypes.c_void_p), blob.nbytes,
+                         None, ctypes.byref(h)) == B.PD_EINVAL
+    assert lib.pd_last_error(None).startswith(b"invalid config: d_model")
 
 
 def _header_text():

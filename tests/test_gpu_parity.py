@@ -30,6 +30,9 @@ pytestmark = pytest.mark.gpu
 # fp32 models, whose logits agree to 1e-4 of the row maximum (|logit| < 2 here).
 MARGIN_BF16 = 0.05
 MARGIN_F32 = 1e-3
+# Fraction of positions whose oracle margin clears MARGIN_BF16 on the Marian-sized model's
+# greedy output (printed by the tests that check it).
+MARIAN_MIN_COVERED = 0.3
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -61,14 +64,24 @@ class Setup:
             self._mem[key] = self.model.encode(np.asarray(src))
         return self._mem[key]
 
-    def step(self, src):
+    def step(self, src, record=None):
+        """The oracle pass; with ``record`` (a list) every call appends the largest |logit| of
+        each of its rows, so that a run's k-th pass can be matched with its logit scale."""
         mem = self.mem(src)
         model = self.model
 
         def step(inputs):
-            idx, margin, prob = om.top2(model.logits(mem, np.asarray(inputs)))
+            lg = model.logits(mem, np.asarray(inputs))
+            if record is not None:
+                record.append(np.abs(lg).max(axis=1))
+            idx, margin, prob = om.top2(lg)
             return od.StepOut(idx, margin, prob)
         return step
+
+    @property
+    def bar(self):
+        """Parity bar on logits: |gpu - oracle| <= bar * max |oracle logit| of the row."""
+        return 2e-2 if self.spec.dtype == synth.DTYPE_BF16 else 1e-4
 
 
 @pytest.fixture(scope="module")
@@ -114,6 +127,23 @@ def tiny_fast():
     s.dec.close()
 
 
+# A bf16 model with the Marian structure (post-LN, SiLU) at a small size whose predictions
+# depend on position and source more than on the previous token (token-embedding scale 0.012,
+# LayerNorm gains and biases perturbed by N(0, 1)): blocks converge in fewer passes than they
+# have positions, and every decision of the oracle's runs on the test sentences clears the
+# bf16 margin 0.05 (smallest about 0.2), so its pass counts and traces are always compared.
+BF16_KNOB = synth.small_spec("post-silu-bf16-knob", d_model=512, n_heads=8, d_ff=1024,
+                             n_enc_layers=2, n_dec_layers=3, vocab=1000,
+                             activation=synth.ACT_SILU, max_pos=128, dtype=synth.DTYPE_BF16)
+
+
+@pytest.fixture(scope="module")
+def bf16_knob():
+    s = Setup(BF16_KNOB, 64, 64, seed=12, ln_noise=1.0, embed_std=0.012)
+    yield s
+    s.dec.close()
+
+
 @pytest.fixture(scope="module")
 def marian():
     s = Setup(synth.MARIAN, 64, 128, seed=0)
@@ -146,8 +176,29 @@ def all_methods(dec, max_len, stop_at_eos=True):
     return out
 
 
-def assert_same_run(got, ref, name):
-    """GPU run == oracle run: tokens, pass count, and every trace row with its tokens."""
+# Slack of the GPU's log p(top-1) for its own logits: the softmax denominator is an fp32 sum
+# of at most a few hundred terms per chain (per-lane runs, then the CTA and grid merges), whose
+# relative rounding stays far below 1e-4.
+LOGP_SLACK = 1e-4
+
+
+def check_probs(gpu_p, ref_p, row_scale, bar, what):
+    """DDGviz probabilities (softmax probability of the argmax token, Section 3.5) against the
+    oracle's.  log p = l_max - logsumexp(l) moves by at most 2 max_j |dl_j| when the logits
+    move by dl (both terms are 1-Lipschitz in the max norm), and the parity bar bounds
+    max_j |dl_j| by bar * max_j |l_j| of the row: so |log p_gpu - log p_ref| <= 2 * bar * scale
+    + the GPU's own rounding."""
+    gpu_p = np.asarray(gpu_p, dtype=np.float64)
+    ref_p = np.asarray(ref_p, dtype=np.float64)
+    assert (gpu_p > 0).all() and (gpu_p <= 1 + 1e-6).all(), what
+    err = np.abs(np.log(gpu_p) - np.log(ref_p))
+    lim = 2 * bar * np.asarray(row_scale) + LOGP_SLACK
+    assert (err <= lim).all(), (what, err.max(), lim[np.argmax(err - lim)])
+
+
+def assert_same_run(got, ref, name, scales=None, bar=None):
+    """GPU run == oracle run: tokens, pass count, and every trace row with its tokens (and,
+    given the oracle's per-pass row logit scales, its probabilities)."""
     assert got.tokens == ref.tokens, name
     assert got.n_iters == ref.n_iters, name
     assert len(got.trace) == len(ref.trace), name
@@ -155,24 +206,31 @@ def assert_same_run(got, ref, name):
         assert (a["step"], a["block_start"], a["block_len"], a["n_converged"], bool(a["stop"]),
                 a["eos_idx"]) == (r.step, r.block_start, r.block_len, r.n_converged, r.stop,
                                   r.eos_idx), (name, t)
-        assert list(got.trace_tokens[t][:a["block_len"]]) == r.tokens, (name, t)
+        blk = a["block_len"]
+        assert list(got.trace_tokens[t][:blk]) == r.tokens, (name, t)
+        if scales is not None and r.probs is not None:
+            i = a["block_start"]
+            check_probs(got.trace_probs[t][:blk], r.probs, scales[t][i - 1:i - 1 + blk], bar,
+                        (name, t))
 
 
 def compare_with_oracle_runs(setup, src, max_len, res):
-    """Pass counts and traces equal the oracle's run where all its decisions had margin."""
-    step = setup.step(src)
+    """Pass counts, traces and trace probabilities equal the oracle's run where all its
+    decisions had margin."""
     e = setup.eos
-    runs = {"greedy": lambda: od.greedy(step, max_len, eos=e),
-            "jacobi": lambda: od.jacobi(step, max_len, eos=e),
-            "gs3": lambda: od.gs_jacobi(step, max_len, 3, eos=e),
-            "gs5": lambda: od.gs_jacobi(step, max_len, 5, eos=e),
-            "hybrid3_0": lambda: od.hybrid_gs_jacobi(step, max_len, 3, eos=e)}
+    runs = {"greedy": lambda st: od.greedy(st, max_len, eos=e),
+            "jacobi": lambda st: od.jacobi(st, max_len, eos=e),
+            "gs3": lambda st: od.gs_jacobi(st, max_len, 3, eos=e),
+            "gs5": lambda st: od.gs_jacobi(st, max_len, 5, eos=e),
+            "hybrid3_0": lambda st: od.hybrid_gs_jacobi(st, max_len, 3, eos=e)}
     compared = 0
     for name, run in runs.items():
-        ref = run()
+        scales = []
+        ref = run(setup.step(src, record=scales))
         if ref.min_margin <= setup.margin:
             continue
-        assert_same_run(res[name], ref, name)
+        assert len(scales) == ref.n_iters
+        assert_same_run(res[name], ref, name, scales, setup.bar)
         compared += 1
     return compared
 
@@ -315,6 +373,54 @@ def test_tiny_eos_paths(tiny_eos):
     assert seen_eos >= 2
 
 
+def test_bf16_traces_against_oracle(bf16_knob):
+    """bf16 weights: pass counts, per-pass traces and DDGviz probabilities of every method equal
+    the oracle's step-by-step runs (all of its decisions clear the bf16 margin), and blocks
+    really converge early (fewer passes than positions)."""
+    s = bf16_knob
+    compared, early = 0, 0
+    for src in synth.sentences(22, 3, 6, 12, s.spec.vocab):
+        max_len = 2 * len(src)
+        s.dec.encode(src)
+        res = all_methods(s.dec, max_len)
+        g = res["greedy"].tokens
+        for k, r in res.items():
+            assert r.tokens == g, k
+        check_tokens_teacher_forced(s, src, g)
+        compared += compare_with_oracle_runs(s, src, max_len, res)
+        early += res["gs5"].n_iters < max_len
+    assert compared == 15
+    assert early == 3
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny_vary", "bf16_knob", "marian"])
+def test_trace_probs_against_own_logits_and_oracle(name, request):
+    """The DDGviz probability of each greedy pass (softmax probability of the argmax, Section
+    3.5) is computed on the device by an online sum of exponentials merged across CTA partials.
+    It must equal, to fp32 rounding, the probability of the GPU's own teacher-forced logits of
+    the same rows (the decode's rows are those rows, bit for bit), and the oracle's within the
+    bound the measured logit error of each row gives: |d log p| <= 2 max_j |dl_j|."""
+    s = request.getfixturevalue(name)
+    for src in synth.sentences(23, 2, 6, 24, s.spec.vocab):
+        max_len = 2 * len(src) if name != "marian" else 12
+        s.dec.encode(src)
+        g = s.dec.decode("greedy", max_len, trace=True)
+        n = len(g.tokens)
+        p_gpu = np.array([g.trace_probs[t][0] for t in range(n)], dtype=np.float64)
+        y_in = np.array([synth.BOS_ID] + g.tokens[:-1], dtype=np.int32)
+        lg = s.dec.debug_logits(y_in).astype(np.float64)
+        assert list(lg.argmax(axis=1)) == g.tokens
+        lse = lg.max(axis=1) + np.log(np.exp(lg - lg.max(axis=1, keepdims=True)).sum(axis=1))
+        p_own = np.exp(lg.max(axis=1) - lse)
+        assert np.abs(np.log(p_gpu) - np.log(p_own)).max() <= LOGP_SLACK
+        ref = s.model.logits(s.mem(src), y_in)
+        _, _, p_ref = om.top2(ref)
+        dl = np.abs(lg - ref).max(axis=1)
+        assert (dl <= s.bar * np.abs(ref).max(axis=1)).all()
+        err = np.abs(np.log(p_gpu) - np.log(p_ref))
+        assert (err <= 2 * dl + LOGP_SLACK).all(), err.max()
+
+
 def test_marian_methods_bit_identical(marian):
     for src in synth.sentences(41, 3, 8, 12, marian.spec.vocab):
         max_len = 2 * len(src)
@@ -325,7 +431,8 @@ def test_marian_methods_bit_identical(marian):
             assert r.tokens == g.tokens, (m, b)
             assert r.n_iters <= max_len
         frac = check_tokens_teacher_forced(marian, src, g.tokens)
-        assert frac > 0.3
+        print(f"marian sentence of {len(src)} ids: {frac:.3f} of positions checked")
+        assert frac >= MARIAN_MIN_COVERED
 
 
 def test_marian_full_size_sampled(marian):
@@ -342,7 +449,8 @@ def test_marian_full_size_sampled(marian):
         assert r.tokens == g.tokens
         assert r.n_iters <= max_len
         frac = check_tokens_teacher_forced(marian, src, r.tokens)
-        assert frac > 0.3
+        print(f"marian sentence {k} ({len(src)} ids): {frac:.3f} of positions checked")
+        assert frac >= MARIAN_MIN_COVERED
 
 
 def test_device_api_matches_host_api(marian):
@@ -498,8 +606,7 @@ def test_pre_ln_models(name, request):
             assert r.n_iters <= max_len, k
         check_tokens_teacher_forced(s, src, g)
         compared += compare_with_oracle_runs(s, src, max_len, res)
-    if s.spec.dtype == synth.DTYPE_F32:
-        assert compared >= 3
+    assert compared >= 3
 
 
 def test_mbart_full_size_sampled():
