@@ -31,8 +31,10 @@ pytestmark = pytest.mark.gpu
 MARGIN_BF16 = 0.05
 MARGIN_F32 = 1e-3
 # Fraction of positions whose oracle margin clears MARGIN_BF16 on the Marian-sized model's
-# greedy output (printed by the tests that check it).
-MARIAN_MIN_COVERED = 0.3
+# greedy output (printed by the tests that check it): 1.000 on every sentence the tests use
+# (random weights make the model copy its input token, with wide top-1 / top-2 gaps), pinned
+# just below so that a logits regression cannot hide behind the margin mask.
+MARIAN_MIN_COVERED = 0.95
 
 
 @pytest.fixture(scope="module", autouse=True)
