@@ -19,8 +19,11 @@
 #include <algorithm>
 #include <vector>
 
+#include <cudaTypedefs.h>
+
 #include "pd.h"
 #include "pd_device.cuh"
+#include "tc_gemm.cuh"
 
 namespace pd {
 
@@ -50,6 +53,11 @@ struct KParams {
 // (ln_bytes, possibly 0).
 struct SmemLayout {
   size_t xs, part, scratch, commit, ln, ln_bytes, total;
+  // bf16 (tensor-core) kernels: weight slots, staged token rows, epilogue tile; all offsets
+  // are relative to the first 1024-byte aligned address of the dynamic shared memory, and
+  // total includes the 1024 bytes of alignment slack
+  size_t ring, bbuf, epi;
+  int ring_slots;
 };
 
 // The commit region: per pass row r (at most D.rows) its new token (-1 for a NaN row) and
@@ -104,9 +112,30 @@ __host__ __device__ inline size_t vec_smem_bytes(const Dims& D, size_t wsize) {
 }
 
 constexpr size_t kSmemMax = 227 * 1024;    // dynamic shared memory of one CTA
+constexpr size_t kSmemStatic = 8 * 1024;   // reserve for the kernels' static shared memory
 
 __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
-  SmemLayout L;
+  SmemLayout L{};
+  if (wsize == 2) {
+    // tensor-core layout: as many weight slots as fit (at most kRingMax), then the vector
+    // copies if they still fit
+    const size_t budget = kSmemMax - kSmemStatic - 1024;
+    const size_t scratch = (size_t)kWarps * (128 + D.max_keys + 4) * sizeof(float);
+    const size_t fixed = kBBytes + kEpiBytes + scratch + commit_bytes(D) + 64;
+    const size_t room = budget > fixed ? (budget - fixed) / kSlotBytes : 0;
+    L.ring_slots = (int)(room < (size_t)kRingMax ? room : (size_t)kRingMax);
+    L.ring = 0;
+    L.bbuf = (size_t)L.ring_slots * kSlotBytes;
+    L.epi = L.bbuf + kBBytes;
+    L.scratch = L.epi + kEpiBytes;
+    L.xs = L.part = L.scratch;
+    L.commit = L.scratch + scratch;
+    L.ln = (L.commit + commit_bytes(D) + 15) / 16 * 16;
+    const size_t all = vec_smem_bytes(D, wsize), ln = ln_elems(D) * wsize;
+    L.ln_bytes = L.ln + all <= budget ? all : (L.ln + ln <= budget && ln <= kVecSmemMax ? ln : 0);
+    L.total = 1024 + L.ln + L.ln_bytes;
+    return L;
+  }
   const int kmax = D.d > D.f ? D.d : D.f;
   L.xs = 0;
   L.part = L.xs + ((size_t)kMTile * kmax * wsize + 15) / 16 * 16;
@@ -339,6 +368,63 @@ __device__ __forceinline__ GemmArgs<W>& smem_args() {
   return s;
 }
 
+// bf16 kernels run their GEMM phases on the tensor cores (tc_gemm.cuh); fp32 kernels on the
+// SIMT path (gemm_phase).
+template <typename W>
+constexpr bool kTensorCores = sizeof(W) == 2;
+
+// The dynamic shared memory the kernels lay out: for the tensor-core layout its first
+// 1024-byte aligned address (128-byte swizzled operands need 1024-byte aligned atoms).
+template <typename W>
+__device__ __forceinline__ unsigned char* smem_base(unsigned char* raw) {
+  if constexpr (kTensorCores<W>) {
+    const uint32_t a = smem_u32(raw);
+    return raw + ((1024u - (a & 1023u)) & 1023u);
+  } else {
+    return raw;
+  }
+}
+
+// Index of decoder pass phase ph among the pass's GEMM phases (6 per layer, then the LM head).
+__device__ __forceinline__ int decoder_gemm_index(int ph, int Ld) {
+  if (ph == 8 * Ld) return 6 * Ld;
+  const int t = ph & 7;
+  return 6 * (ph >> 3) + (t == PH_QKV ? TD_QKV : t == PH_O ? TD_O : t == PH_QC ? TD_QC
+                          : t == PH_OC ? TD_OC : t == PH_FFN1 ? TD_FFN1 : TD_FFN2);
+}
+
+// One GEMM phase; on the tensor-core path a wait that gave up raises the grid's abort flag and
+// PD_ETIMEOUT, so the other CTAs leave their next barrier instead of waiting for this one.
+template <typename W>
+__device__ __forceinline__ bool run_gemm(const KParams<W>& P, const GemmArgs<W>& g,
+                                         const EmbedTabs<W>& T, int gph, unsigned char* smem) {
+  if constexpr (kTensorCores<W>) {
+    const SmemLayout SL = smem_layout(P.D, sizeof(W));
+    const bool ok = tc_gemm_phase<W>(g, T, P.D, gph, static_cast<const CUtensorMap*>(P.B.tmaps),
+                                     smem + SL.ring, smem + SL.bbuf,
+                                     reinterpret_cast<float*>(smem + SL.epi), P.B.red, P.B.cnt);
+    if (!ok && threadIdx.x == 0) {
+      atomicExch(P.B.bar + 1, 1u);
+      atomicCAS(&P.B.st->status, 0, (int)PD_ETIMEOUT);
+    }
+    return ok;
+  } else {
+    gemm_phase<W>(g, T, P.D, smem);
+    return true;
+  }
+}
+
+// Thread 0 of a tensor-core kernel: top up the weight stream (while the CTA waits at a grid
+// barrier, the slots its last phase used have been released).
+template <typename W>
+__device__ __forceinline__ void stream_weights(const KParams<W>& P, unsigned char* smem) {
+  if constexpr (kTensorCores<W>) {
+    if (threadIdx.x == 0)
+      tc_produce<W>(P.D, static_cast<const CUtensorMap*>(P.B.tmaps),
+                    smem + smem_layout(P.D, sizeof(W)).ring, false);
+  }
+}
+
 // One decoder pass over the M rows described in the commit region, followed by the LM head, as
 // a loop over phases separated by grid barriers.  The arguments of the next GEMM phase are
 // written to shared memory by one thread while its CTA waits at the barrier, and the weights
@@ -346,7 +432,7 @@ __device__ __forceinline__ GemmArgs<W>& smem_args() {
 // phases.
 template <typename W>
 __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tgt,
-                         unsigned char* smem) {
+                         unsigned char* smem, bool pass_open) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
   int* status = &B.st->status;
@@ -356,6 +442,9 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
   const EmbedTabs<W> T = embed_tabs(P);
   GemmArgs<W>& ga = smem_args<W>();
   const int nph = 8 * D.Ld + 1;
+  if constexpr (kTensorCores<W>) {
+    if (threadIdx.x == 0) tc_begin_pass<W>(M, pass_open);
+  }
   if (threadIdx.x == 32) gemm_args(P, 0, M, cm.rtok, cm.rpos, cm.rslot, logits, ga);
   prefetch_pass_start(P);
   __syncthreads();
@@ -371,8 +460,8 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
       else
         attn_phase<W, W>(D, B.q, B.kcross + l * cross_ld, B.vcross + l * cross_ld, B.att, M,
                          cm.rxb, cm.rxn, 0, scratch);
-    } else {
-      gemm_phase<W>(ga, T, D, smem);
+    } else if (!run_gemm<W>(P, ga, T, decoder_gemm_index(ph, D.Ld), smem)) {
+      return false;
     }
     if (ph == nph - 1) break;            // the caller's barrier follows the LM head
     const int next = is_attn_phase(ph + 1, nph) ? ph + 2 : ph + 1;
@@ -380,6 +469,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
           if (!attn && threadIdx.x == 32)
             gemm_args(P, next, M, cm.rtok, cm.rpos, cm.rslot, logits, ga);
           prefetch_phase(P, ph + 3);
+          stream_weights(P, smem);
         }))
       return false;
   }
@@ -591,7 +681,8 @@ __device__ void write_outputs(const KParams<W>& P, unsigned char* smem) {
 
 template <typename W>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
-  extern __shared__ __align__(16) unsigned char smem[];
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  unsigned char* smem = smem_base<W>(smem_raw);
   unsigned tgt = 0;
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
@@ -600,6 +691,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   load_smem_vectors<W>(D, smem);
   const SmemLayout SL = smem_layout(D, sizeof(W));
   const CommitMem cm = commit_mem(D, smem + SL.commit);
+  if constexpr (kTensorCores<W>) tc_setup<W>(D, TC_DECODE, SL.ring_slots);
 
   if (P.debug_len > 0) {                  // teacher-forced rows 0..len-1 of the slot-0 sentence
     for (int m = threadIdx.x; m < P.debug_len; m += blockDim.x) {
@@ -608,7 +700,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
       cm.rxb[m] = 0; cm.rxn[m] = P.n_src_s[0];
     }
     __syncthreads();
-    run_pass<W>(P, P.debug_len, P.logits, tgt, smem);
+    run_pass<W>(P, P.debug_len, P.logits, tgt, smem, false);
+    if constexpr (kTensorCores<W>) tc_teardown<W>();
     return;
   }
 
@@ -636,20 +729,21 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   for (;;) {
     const int M = cm.misc[0];
     if (M == 0) break;
-    if (!run_pass<W>(P, M, nullptr, tgt, smem)) break;
-    if (!grid_barrier(B.bar, tgt, status)) break;
+    if (!run_pass<W>(P, M, nullptr, tgt, smem, true)) break;
+    if (!grid_barrier(B.bar, tgt, status, [&] { stream_weights(P, smem); })) break;
     commit<W>(P, smem);
   }
   if (blockIdx.x == 0) write_outputs(P, smem);
+  if constexpr (kTensorCores<W>) tc_teardown<W>();
 }
 
+// The encoder pass of encode_kernel: every encoder layer (QKV, full self-attention, O, FFN1,
+// FFN2, phases separated by grid barriers), then the cross-attention keys and values of every
+// decoder layer from the encoder output.  False if a barrier or a wait gave up.
 template <typename W>
-__global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
-  extern __shared__ __align__(16) unsigned char smem[];
-  unsigned tgt = 0;
+__device__ bool encode_pass(const KParams<W>& P, unsigned char* smem, unsigned& tgt) {
   const Dims& D = P.D;
   const Bufs<W>& B = P.B;
-  load_smem_mw(P);
   const ModelW<W>& mw = smem_mw<W>();
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
@@ -659,6 +753,9 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
   const int n = P.n_src;
   const CommitMem cm = commit_mem(D, smem + SL.commit);
   for (int m = threadIdx.x; m < n; m += blockDim.x) cm.rpos[m] = m;   // source positions
+  if constexpr (kTensorCores<W>) {
+    if (threadIdx.x == 0) tc_begin_pass<W>(n, false);
+  }
   __syncthreads();
 
   for (int l = 0; l < D.Le; ++l) {
@@ -669,6 +766,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     prefetch_gemm_weights(L.w2, D.d, D.f);
   }
   for (int l = 0; l < D.Ld; ++l) prefetch_gemm_weights(mw.dec[l].wkvc, 2 * D.d, D.d);
+  auto barrier = [&] { return grid_barrier(B.bar, tgt, status, [&] { stream_weights(P, smem); }); };
 
   for (int l = 0; l < D.Le; ++l) {
     const EncLayerW<W>& L = mw.enc[l];
@@ -686,18 +784,16 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
     g.kdst_f = B.k; g.vdst_f = B.v;
     gemm_plan(g, gridDim.x);
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return;
+    if (!run_gemm<W>(P, g, T, 4 * l + TE_QKV, smem) || !barrier()) return false;
 
     attn_phase<float, W>(D, B.q, B.k, B.v, B.att, n, nullptr, nullptr, n, scratch);
-    if (!grid_barrier(B.bar, tgt, status)) return;
+    if (!barrier()) return false;
 
     g = GemmArgs<W>{};
     g.M = n; g.N = D.d; g.K = D.d; g.xw_src = B.att; g.w = L.wo; g.bias = L.bo;
     g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
     gemm_plan(g, gridDim.x);
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return;
+    if (!run_gemm<W>(P, g, T, 4 * l + TE_O, smem) || !barrier()) return false;
 
     g = GemmArgs<W>{};
     g.M = n; g.N = D.f; g.K = D.d; g.x_src = B.rb;
@@ -706,18 +802,16 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     const float* res2 = pre ? B.rb : B.xb;
     g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out_w = B.ffh; g.ld = D.f;
     gemm_plan(g, gridDim.x);
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return;
+    if (!run_gemm<W>(P, g, T, 4 * l + TE_FFN1, smem) || !barrier()) return false;
 
     g = GemmArgs<W>{};
     g.M = n; g.N = D.d; g.K = D.f; g.xw_src = B.ffh; g.w = L.w2; g.bias = L.b2;
     g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res2;
     gemm_plan(g, gridDim.x);
-    gemm_phase<W>(g, T, D, smem);
-    if (!grid_barrier(B.bar, tgt, status)) return;
+    if (!run_gemm<W>(P, g, T, 4 * l + TE_FFN2, smem) || !barrier()) return false;
   }
   // cross-attention keys and values of every decoder layer from the encoder output, into the
-  // sentence's slot
+  // sentence's slot (independent phases: no barrier between them)
   const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
   const size_t slot_off = (size_t)P.enc_slot * D.max_src * D.d;
   for (int l = 0; l < D.Ld; ++l) {
@@ -729,8 +823,20 @@ __global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
     g.kdst = B.kcross + l * cross_ld + slot_off;
     g.vdst = B.vcross + l * cross_ld + slot_off;
     gemm_plan(g, gridDim.x);
-    gemm_phase<W>(g, T, D, smem);
+    if (!run_gemm<W>(P, g, T, 4 * D.Le + l, smem)) return false;
   }
+  return true;
+}
+
+template <typename W>
+__global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  unsigned char* smem = smem_base<W>(smem_raw);
+  unsigned tgt = 0;
+  load_smem_mw(P);
+  if constexpr (kTensorCores<W>) tc_setup<W>(P.D, TC_ENCODE, smem_layout(P.D, sizeof(W)).ring_slots);
+  (void)encode_pass<W>(P, smem, tgt);
+  if constexpr (kTensorCores<W>) tc_teardown<W>();
 }
 
 }  // namespace pd
@@ -802,6 +908,8 @@ bool valid_config(const pd_config* c, std::string* why) {
     if (id < 0 || id >= c->vocab) return bad("special ids must be in [0, vocab)");
   if (!(c->ln_eps >= 0.f)) return bad("ln_eps");
   if (c->max_batch < 0 || c->max_batch > pd::kMaxBatch) return bad("max_batch must be in [0, 64]");
+  if (c->dtype == PD_DTYPE_BF16 && c->vocab < pd::kTileN)
+    return bad("bf16 models need vocab >= 128 (one tensor-core tile)");
   return true;
 }
 
@@ -879,6 +987,85 @@ pd_status raise_smem_limit(pd_ctx* c, const void* fn) {
   return PD_OK;
 }
 
+// cuTensorMapEncodeTiled from the driver (through the runtime's entry-point query, so the
+// library needs no link against the driver library).
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Tensor-core resources of a bf16 context: a TMA tensor map per weight matrix ([N][K] bf16,
+// boxes of 128 rows x 64 K elements with the 128-byte swizzle the MMA's shared-memory
+// descriptors expect; rows past N read as zero), the split-K partial buffer and its arrival
+// counters.
+pd_status tc_resources(pd_ctx* c, const pd::ModelW<__nv_bfloat16>& mw) {
+  const Dims& D = c->D;
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return fail(c, PD_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  std::vector<CUtensorMap> maps(pd::kNumTmaps);
+  std::memset(maps.data(), 0, maps.size() * sizeof(CUtensorMap));
+  auto make = [&](int idx, const __nv_bfloat16* w, int N, int K) -> pd_status {
+    cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)N};
+    cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    cuuint32_t box[2] = {(cuuint32_t)pd::kKBlock, (cuuint32_t)pd::kTileN};
+    cuuint32_t estr[2] = {1, 1};
+    const CUresult r = enc(&maps[idx], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                           const_cast<__nv_bfloat16*>(w), dims, strides, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(c, PD_ECUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
+    return PD_OK;
+  };
+  const int d = D.d, f = D.f;
+  for (int l = 0; l < D.Le; ++l) {
+    const auto& L = mw.enc[l];
+    PD_TRY(make(4 * l + 0, L.wqkv, 3 * d, d));
+    PD_TRY(make(4 * l + 1, L.wo, d, d));
+    PD_TRY(make(4 * l + 2, L.w1, f, d));
+    PD_TRY(make(4 * l + 3, L.w2, d, f));
+  }
+  for (int l = 0; l < D.Ld; ++l) {
+    const auto& L = mw.dec[l];
+    const int b = pd::kTmapDec + 7 * l;
+    PD_TRY(make(b + 0, L.wqkv, 3 * d, d));
+    PD_TRY(make(b + 1, L.wo, d, d));
+    PD_TRY(make(b + 2, L.wqc, d, d));
+    PD_TRY(make(b + 3, L.woc, d, d));
+    PD_TRY(make(b + 4, L.w1, f, d));
+    PD_TRY(make(b + 5, L.w2, d, f));
+    PD_TRY(make(b + 6, L.wkvc, 2 * d, d));
+  }
+  PD_TRY(make(pd::kTmapEmbed, mw.embed, D.V, d));
+  CUtensorMap* dmaps = nullptr;
+  PD_TRY(dalloc(c, &dmaps, maps.size()));
+  PD_CUDA(c, cudaMemcpy(dmaps, maps.data(), maps.size() * sizeof(CUtensorMap),
+                        cudaMemcpyHostToDevice));
+  // the largest split-K partial buffer any GEMM phase needs: S x N x rows floats
+  size_t red = 1;
+  for (int kind : {pd::TC_DECODE, pd::TC_ENCODE})
+    for (int g = 0; g < pd::gemm_phase_count(D, kind); ++g) {
+      const pd::Geom G = pd::gemm_geom(D, kind, g);
+      if (G.S > 1) red = std::max(red, (size_t)G.S * G.N * D.rows);
+    }
+  pd::Bufs<__nv_bfloat16>& B = c->bb;
+  B.tmaps = dmaps;
+  PD_TRY(dalloc(c, &B.red, red));
+  PD_TRY(dalloc(c, &B.cnt, (size_t)pd::kCounterSlots));
+  PD_CUDA(c, cudaMemset(B.cnt, 0, pd::kCounterSlots * sizeof(unsigned)));
+  return PD_OK;
+}
+pd_status tc_resources(pd_ctx*, const pd::ModelW<float>&) { return PD_OK; }
+
 template <typename W>
 pd_status create_impl(pd_ctx* c, const void* weights) {
   const pd_config& cfg = c->cfg;
@@ -939,7 +1126,12 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
   PD_CUDA(c, cudaMemset(B.st, 0, sizeof(pd::DecState)));
   PD_CUDA(c, cudaMemset(B.bar, 0, 4 * sizeof(unsigned)));
 
+  if constexpr (sizeof(W) == 2) PD_TRY(tc_resources(c, mw));
+
   c->smem = pd::smem_layout(D, sizeof(W)).total;
+  if (sizeof(W) == 2 && pd::smem_layout(D, sizeof(W)).ring_slots < 2)
+    return fail(c, PD_EINVAL, "the tensor-core kernels' shared memory does not fit (max_tgt_len "
+                              "or max_batch too large)");
   // the limit is per kernel function and shared by every context of the process: only raise it
   PD_TRY(raise_smem_limit(c, (const void*)pd::decode_kernel<W>));
   PD_TRY(raise_smem_limit(c, (const void*)pd::encode_kernel<W>));

@@ -108,6 +108,9 @@ struct Bufs {
   int* src;                    // [max_src]
   int* dbg_tok;                // [max_tgt]
   float* pos_tab;              // sinusoidal positions [rows][d] (built once at create)
+  const void* tmaps;           // bf16: CUtensorMap of every weight matrix (device memory)
+  float* red;                  // bf16: split-K partial sums [S][rows][N]
+  unsigned* cnt;               // bf16: split-K arrival counters (zero between uses)
 };
 
 // ------------------------------------------------------------------------------------------

@@ -287,6 +287,22 @@ def test_marian_logits_bf16(marian):
         assert rel_row_err(got, ref).max() < 2e-2
 
 
+@pytest.mark.parametrize("name", ["tiny", "bf16_knob", "marian"])
+def test_logits_batch_invariant(name, request):
+    """Batch invariance, the property behind every method's bit identity with greedy: the
+    logits of row t (inputs y_0..y_t) are the same bits whether the pass carries t + 1 rows or
+    more, whatever MMA tile, chunk or slot the row falls in (passes of 1 to 40 rows)."""
+    s = request.getfixturevalue(name)
+    rng = np.random.default_rng(13)
+    src = rng.integers(3, s.spec.vocab, size=19).astype(np.int32)
+    y_in = np.r_[synth.BOS_ID, rng.integers(3, s.spec.vocab, size=39)].astype(np.int32)
+    s.dec.encode(src)
+    full = s.dec.debug_logits(y_in)
+    for T in (1, 5, 16, 17, 33):
+        part = s.dec.debug_logits(y_in[:T])
+        assert np.array_equal(part.view(np.uint32), full[:T].view(np.uint32)), T
+
+
 # ---- tokens, bit identity, traces ------------------------------------------------------------
 
 @pytest.mark.parametrize("name", ["tiny", "tiny_ln", "tiny_vary", "tiny_eos"])
