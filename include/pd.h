@@ -73,7 +73,20 @@ typedef struct {
   int max_tgt_len;   /* capacity: largest max_len pd_decode accepts */
   int max_batch;     /* capacity: sentences one pd_encode_batch / pd_decode_batch carries,
                         0 or 1..64 (0 = 1); each needs its own key/value caches */
+  int gemm_engine;   /* pd_gemm_engine: how the bf16 matrix products run (fp32: always SIMT) */
 } pd_config;
+
+/* How a bf16 context runs the matrix products of its encoder and decoder passes.  Every pass of
+ * a context uses the same engine, so each row's arithmetic is the same whatever the pass
+ * carries and every decoding method returns exactly the context's greedy tokens; the two
+ * engines round differently (both within the bf16 parity bar).
+ *  PD_ENGINE_SIMT: CUDA-core dot products spread over every SM; the latency-bound choice for
+ *    passes of a few rows (one sentence, small blocks).
+ *  PD_ENGINE_TENSOR: 5th-generation tensor cores (tcgen05, accumulators in tensor memory),
+ *    weight tiles streamed by TMA; the choice when passes carry many rows (batched serving,
+ *    full-sentence Jacobi).
+ *  PD_ENGINE_AUTO: TENSOR when max_batch > 1, else SIMT. */
+typedef enum { PD_ENGINE_AUTO = 0, PD_ENGINE_SIMT = 1, PD_ENGINE_TENSOR = 2 } pd_gemm_engine;
 
 typedef struct pd_ctx pd_ctx;
 

@@ -23,6 +23,7 @@ STATUS_NAMES = {0: "PD_OK", -1: "PD_EINVAL", -2: "PD_ENOMEM", -3: "PD_ECUDA", -4
 
 METHODS = {"greedy": 0, "jacobi": 1, "gs_jacobi": 2, "hybrid_gs_jacobi": 3}
 STOP_RULES = {"paper": 0, "prefix": 1}      # pd_stop_rule: Eq. 5 StopC, accepted prefix
+ENGINES = {"auto": 0, "simt": 1, "tensor": 2}   # pd_gemm_engine
 
 # Every symbol include/pd.h declares.
 EXPORTED = ("pd_weights_nbytes", "pd_create", "pd_export_weights", "pd_encode",
@@ -44,7 +45,8 @@ class _Config(ctypes.Structure):
                                             "learned_pos", "max_pos", "dtype", "pad_id",
                                             "eos_id", "bos_id")] + \
               [("ln_eps", ctypes.c_float), ("max_src_len", ctypes.c_int),
-               ("max_tgt_len", ctypes.c_int), ("max_batch", ctypes.c_int)]
+               ("max_tgt_len", ctypes.c_int), ("max_batch", ctypes.c_int),
+               ("gemm_engine", ctypes.c_int)]
 
 
 class _DecodeParams(ctypes.Structure):
@@ -135,15 +137,16 @@ class Config:
     max_src_len: int = 128
     max_tgt_len: int = 256
     max_batch: int = 0
+    gemm_engine: int = 0
 
     @classmethod
     def from_spec(cls, spec, max_src_len: int, max_tgt_len: int, pad_id=1, eos_id=0, bos_id=2,
-                  max_batch: int = 0):
+                  max_batch: int = 0, engine: str = "auto"):
         """Build from any object carrying the model fields (d_model, n_heads, ...)."""
         return cls(spec.d_model, spec.n_heads, spec.d_ff, spec.n_enc_layers, spec.n_dec_layers,
                    spec.vocab, spec.activation, bool(spec.pre_ln), bool(spec.learned_pos),
                    spec.max_pos, spec.dtype, pad_id, eos_id, bos_id, spec.ln_eps, max_src_len,
-                   max_tgt_len, max_batch)
+                   max_tgt_len, max_batch, ENGINES[engine])
 
     def _c(self) -> _Config:
         c = _Config()

@@ -44,6 +44,8 @@ struct KParams {
   int32_t* out_y;           // [n_sent][out_ld]
   int out_ld;
   int32_t* out_info;        // [n_sent][4] = {n_y, n_iters, status, n_trace}
+  // bf16: TMA tensor map of the weight matrix of every GEMM phase of this kernel's sequence
+  CUtensorMap maps[kMaxKernelMaps];
 };
 
 // Dynamic shared memory of the decode / encode kernels (byte offsets): xs, the staged GEMM
@@ -116,7 +118,7 @@ constexpr size_t kSmemStatic = 8 * 1024;   // reserve for the kernels' static sh
 
 __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   SmemLayout L{};
-  if (wsize == 2) {
+  if (wsize == 2 && D.tc) {
     // tensor-core layout: as many weight slots as fit (at most kRingMax), then the vector
     // copies if they still fit
     const size_t budget = kSmemMax - kSmemStatic - 1024;
@@ -144,8 +146,11 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
   L.ln = (L.commit + commit_bytes(D) + 15) / 16 * 16;
   // the vector copies are kept only when they fit beside the rest
   const size_t all = vec_smem_bytes(D, wsize), ln = ln_elems(D) * wsize;
-  L.ln_bytes = L.ln + all <= kSmemMax ? all : (L.ln + ln <= kSmemMax && ln <= kVecSmemMax ? ln : 0);
-  L.total = L.ln + L.ln_bytes;
+  // bf16 kernels align their dynamic shared memory to 1024 bytes (smem_base): keep the slack
+  const size_t slack = wsize == 2 ? 1024 : 0;
+  L.ln_bytes = L.ln + all + slack <= kSmemMax ? all
+               : (L.ln + ln + slack <= kSmemMax && ln <= kVecSmemMax ? ln : 0);
+  L.total = slack + L.ln + L.ln_bytes;
   return L;
 }
 
@@ -161,12 +166,32 @@ __device__ __forceinline__ ModelW<W>& smem_mw() {
   __shared__ ModelW<W> s;
   return s;
 }
+// The model dimensions, also copied into shared memory: device functions that are not inlined
+// take them by reference, and a reference into the kernel parameters or the stack would be
+// read through L1, which every barrier's acquire drops.
+template <typename W>
+__device__ __forceinline__ Dims& smem_dims() {
+  __shared__ Dims s;
+  return s;
+}
+template <typename W>
+__device__ __forceinline__ EmbedTabs<W>& smem_tabs() {
+  __shared__ EmbedTabs<W> s;
+  return s;
+}
 template <typename W>
 __device__ __forceinline__ void load_smem_mw(const KParams<W>& P) {
   static_assert(sizeof(ModelW<W>) % 8 == 0, "pointer table");
   const unsigned long long* src = reinterpret_cast<const unsigned long long*>(P.mw);
   unsigned long long* dst = reinterpret_cast<unsigned long long*>(&smem_mw<W>());
   for (int i = threadIdx.x; i < (int)(sizeof(ModelW<W>) / 8); i += blockDim.x) dst[i] = src[i];
+  if (threadIdx.x == 0) smem_dims<W>() = P.D;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const ModelW<W>& mw = smem_mw<W>();
+    smem_tabs<W>() = EmbedTabs<W>{mw.embed, P.D.learned_pos ? mw.pos : nullptr,
+                                  P.D.learned_pos ? nullptr : P.B.pos_tab};
+  }
   __syncthreads();
 }
 
@@ -243,13 +268,6 @@ __device__ void load_smem_vectors(const Dims& D, unsigned char* smem) {
   __syncthreads();
 }
 
-template <typename W>
-__device__ __forceinline__ EmbedTabs<W> embed_tabs(const KParams<W>& P) {
-  const ModelW<W>& mw = smem_mw<W>();
-  return EmbedTabs<W>{mw.embed, P.D.learned_pos ? mw.pos : nullptr,
-                      P.D.learned_pos ? nullptr : P.B.pos_tab};
-}
-
 // Phases of a decoder pass, per layer in this order (the attention phases take scalar
 // arguments); phase 8 * Ld is the LM head.
 enum : int {
@@ -266,7 +284,7 @@ __device__ __forceinline__ bool is_attn_phase(int ph, int nph) {
 template <typename W>
 __device__ void gemm_args(const KParams<W>& P, int ph, int M, const int* rtok, const int* rpos,
                           const int* rslot, float* logits, GemmArgs<W>& g) {
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const Bufs<W>& B = P.B;
   const ModelW<W>& mw = smem_mw<W>();
   const bool pre = D.pre_ln != 0;
@@ -337,7 +355,7 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, const int* rtok, c
 // so that HBM streams them while the latency-bound chain of earlier phases runs.
 template <typename W>
 __device__ void prefetch_phase(const KParams<W>& P, int ph) {
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const int nph = 8 * D.Ld + 1;
   if (ph >= nph || is_attn_phase(ph, nph)) return;
   const ModelW<W>& mw = smem_mw<W>();
@@ -359,7 +377,7 @@ template <typename W>
 __device__ void prefetch_pass_start(const KParams<W>& P) {
   prefetch_phase(P, 0);
   prefetch_phase(P, 2);
-  prefetch_phase(P, 8 * P.D.Ld);
+  prefetch_phase(P, 8 * smem_dims<W>().Ld);
 }
 
 template <typename W>
@@ -368,10 +386,12 @@ __device__ __forceinline__ GemmArgs<W>& smem_args() {
   return s;
 }
 
-// bf16 kernels run their GEMM phases on the tensor cores (tc_gemm.cuh); fp32 kernels on the
-// SIMT path (gemm_phase).
+// bf16 kernels can run their GEMM phases on the tensor cores (tc_gemm.cuh), as the context
+// chose (Dims::tc); fp32 kernels always run them on the SIMT path (gemm_phase).
 template <typename W>
 constexpr bool kTensorCores = sizeof(W) == 2;
+// Kernels are instantiated per engine (TC): the SIMT instantiation carries no tensor-core code,
+// so the register allocation of its GEMM phase is the one it was tuned with.
 
 // The dynamic shared memory the kernels lay out: for the tensor-core layout its first
 // 1024-byte aligned address (128-byte swizzled operands need 1024-byte aligned atoms).
@@ -395,12 +415,13 @@ __device__ __forceinline__ int decoder_gemm_index(int ph, int Ld) {
 
 // One GEMM phase; on the tensor-core path a wait that gave up raises the grid's abort flag and
 // PD_ETIMEOUT, so the other CTAs leave their next barrier instead of waiting for this one.
-template <typename W>
+template <typename W, bool TC>
 __device__ __forceinline__ bool run_gemm(const KParams<W>& P, const GemmArgs<W>& g,
                                          const EmbedTabs<W>& T, int gph, unsigned char* smem) {
-  if constexpr (kTensorCores<W>) {
-    const SmemLayout SL = smem_layout(P.D, sizeof(W));
-    const bool ok = tc_gemm_phase<W>(g, T, P.D, gph, static_cast<const CUtensorMap*>(P.B.tmaps),
+  if constexpr (TC) {
+    const Dims& D = smem_dims<W>();
+    const SmemLayout SL = smem_layout(D, sizeof(W));
+    const bool ok = tc_gemm_phase<W>(g, T, D, gph, P.maps,
                                      smem + SL.ring, smem + SL.bbuf,
                                      reinterpret_cast<float*>(smem + SL.epi), P.B.red, P.B.cnt);
     if (!ok && threadIdx.x == 0) {
@@ -409,19 +430,19 @@ __device__ __forceinline__ bool run_gemm(const KParams<W>& P, const GemmArgs<W>&
     }
     return ok;
   } else {
-    gemm_phase<W>(g, T, P.D, smem);
+    gemm_phase<W>(g, T, smem_dims<W>(), smem);
     return true;
   }
 }
 
 // Thread 0 of a tensor-core kernel: top up the weight stream (while the CTA waits at a grid
 // barrier, the slots its last phase used have been released).
-template <typename W>
+template <typename W, bool TC>
 __device__ __forceinline__ void stream_weights(const KParams<W>& P, unsigned char* smem) {
-  if constexpr (kTensorCores<W>) {
+  if constexpr (TC) {
     if (threadIdx.x == 0)
-      tc_produce<W>(P.D, static_cast<const CUtensorMap*>(P.B.tmaps),
-                    smem + smem_layout(P.D, sizeof(W)).ring, false);
+      tc_produce<W>(smem_dims<W>(), P.maps,
+                    smem + smem_layout(smem_dims<W>(), sizeof(W)).ring, false);
   }
 }
 
@@ -430,23 +451,25 @@ __device__ __forceinline__ void stream_weights(const KParams<W>& P, unsigned cha
 // written to shared memory by one thread while its CTA waits at the barrier, and the weights
 // three phases ahead are requested from L2 there, so that neither is on the chain of dependent
 // phases.
-template <typename W>
+template <typename W, bool TC>
 __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tgt,
                          unsigned char* smem, bool pass_open) {
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const Bufs<W>& B = P.B;
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
   const CommitMem cm = commit_mem(D, smem + SL.commit);
-  const EmbedTabs<W> T = embed_tabs(P);
+  const EmbedTabs<W>& T = smem_tabs<W>();
   GemmArgs<W>& ga = smem_args<W>();
   const int nph = 8 * D.Ld + 1;
-  if constexpr (kTensorCores<W>) {
+  if constexpr (TC) {
     if (threadIdx.x == 0) tc_begin_pass<W>(M, pass_open);
   }
   if (threadIdx.x == 32) gemm_args(P, 0, M, cm.rtok, cm.rpos, cm.rslot, logits, ga);
-  prefetch_pass_start(P);
+  // the SIMT path asks L2 for the weights ahead; the tensor-core path streams them itself (its
+  // TMA loads would queue behind bulk L2 prefetches in the same copy engine)
+  if constexpr (!TC) prefetch_pass_start(P);
   __syncthreads();
   const size_t self_ld = (size_t)D.max_batch * D.max_tgt * D.d;
   const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
@@ -460,7 +483,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
       else
         attn_phase<W, W>(D, B.q, B.kcross + l * cross_ld, B.vcross + l * cross_ld, B.att, M,
                          cm.rxb, cm.rxn, 0, scratch);
-    } else if (!run_gemm<W>(P, ga, T, decoder_gemm_index(ph, D.Ld), smem)) {
+    } else if (!run_gemm<W, TC>(P, ga, T, decoder_gemm_index(ph, D.Ld), smem)) {
       return false;
     }
     if (ph == nph - 1) break;            // the caller's barrier follows the LM head
@@ -468,8 +491,8 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
     if (!grid_barrier(B.bar, tgt, status, [&] {
           if (!attn && threadIdx.x == 32)
             gemm_args(P, next, M, cm.rtok, cm.rpos, cm.rslot, logits, ga);
-          prefetch_phase(P, ph + 3);
-          stream_weights(P, smem);
+          if constexpr (!TC) prefetch_phase(P, ph + 3);
+          stream_weights<W, TC>(P, smem);
         }))
       return false;
   }
@@ -485,7 +508,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
 // note), sentences in order.  All threads of the CTA; misc[0] = the row count.
 template <typename W>
 __device__ void build_rows(const KParams<W>& P, const CommitMem& cm) {
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const int S = P.n_sent;
   if (threadIdx.x == 0) {
     int r = 0;
@@ -522,7 +545,7 @@ __device__ void build_rows(const KParams<W>& P, const CommitMem& cm) {
 // decodes).  Ends with the rows of the next pass.
 template <typename W>
 __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const Bufs<W>& B = P.B;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   const CommitMem cm = commit_mem(D, smem + SL.commit);
@@ -652,7 +675,7 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
 // precedence.
 template <typename W>
 __device__ void write_outputs(const KParams<W>& P, unsigned char* smem) {
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const SmemLayout SL = smem_layout(D, sizeof(W));
   const CommitMem cm = commit_mem(D, smem + SL.commit);
   const int S = P.n_sent;
@@ -679,19 +702,19 @@ __device__ void write_outputs(const KParams<W>& P, unsigned char* smem) {
 // kernels
 // ------------------------------------------------------------------------------------------
 
-template <typename W>
-__global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
+template <typename W, bool TC>
+__global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ KParams<W> P) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   unsigned char* smem = smem_base<W>(smem_raw);
   unsigned tgt = 0;
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const Bufs<W>& B = P.B;
   int* status = &B.st->status;
   load_smem_mw(P);
   load_smem_vectors<W>(D, smem);
   const SmemLayout SL = smem_layout(D, sizeof(W));
   const CommitMem cm = commit_mem(D, smem + SL.commit);
-  if constexpr (kTensorCores<W>) tc_setup<W>(D, TC_DECODE, SL.ring_slots);
+  if constexpr (TC) tc_setup<W>(D, TC_DECODE, SL.ring_slots, P.maps);
 
   if (P.debug_len > 0) {                  // teacher-forced rows 0..len-1 of the slot-0 sentence
     for (int m = threadIdx.x; m < P.debug_len; m += blockDim.x) {
@@ -700,8 +723,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
       cm.rxb[m] = 0; cm.rxn[m] = P.n_src_s[0];
     }
     __syncthreads();
-    run_pass<W>(P, P.debug_len, P.logits, tgt, smem, false);
-    if constexpr (kTensorCores<W>) tc_teardown<W>();
+    run_pass<W, TC>(P, P.debug_len, P.logits, tgt, smem, false);
+    if constexpr (TC) tc_teardown<W>();
     return;
   }
 
@@ -729,44 +752,46 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(KParams<W> P) {
   for (;;) {
     const int M = cm.misc[0];
     if (M == 0) break;
-    if (!run_pass<W>(P, M, nullptr, tgt, smem, true)) break;
-    if (!grid_barrier(B.bar, tgt, status, [&] { stream_weights(P, smem); })) break;
+    if (!run_pass<W, TC>(P, M, nullptr, tgt, smem, true)) break;
+    if (!grid_barrier(B.bar, tgt, status, [&] { stream_weights<W, TC>(P, smem); })) break;
     commit<W>(P, smem);
   }
   if (blockIdx.x == 0) write_outputs(P, smem);
-  if constexpr (kTensorCores<W>) tc_teardown<W>();
+  if constexpr (TC) tc_teardown<W>();
 }
 
 // The encoder pass of encode_kernel: every encoder layer (QKV, full self-attention, O, FFN1,
 // FFN2, phases separated by grid barriers), then the cross-attention keys and values of every
 // decoder layer from the encoder output.  False if a barrier or a wait gave up.
-template <typename W>
+template <typename W, bool TC>
 __device__ bool encode_pass(const KParams<W>& P, unsigned char* smem, unsigned& tgt) {
-  const Dims& D = P.D;
+  const Dims& D = smem_dims<W>();
   const Bufs<W>& B = P.B;
   const ModelW<W>& mw = smem_mw<W>();
   int* status = &B.st->status;
   const SmemLayout SL = smem_layout(D, sizeof(W));
   float* scratch = reinterpret_cast<float*>(smem + SL.scratch);
-  const EmbedTabs<W> T = embed_tabs(P);
+  const EmbedTabs<W>& T = smem_tabs<W>();
   const bool pre = D.pre_ln != 0;
   const int n = P.n_src;
   const CommitMem cm = commit_mem(D, smem + SL.commit);
   for (int m = threadIdx.x; m < n; m += blockDim.x) cm.rpos[m] = m;   // source positions
-  if constexpr (kTensorCores<W>) {
+  if constexpr (TC) {
     if (threadIdx.x == 0) tc_begin_pass<W>(n, false);
   }
   __syncthreads();
 
-  for (int l = 0; l < D.Le; ++l) {
-    const EncLayerW<W>& L = mw.enc[l];
-    prefetch_gemm_weights(L.wqkv, 3 * D.d, D.d);
-    prefetch_gemm_weights(L.wo, D.d, D.d);
-    prefetch_gemm_weights(L.w1, D.f, D.d);
-    prefetch_gemm_weights(L.w2, D.d, D.f);
+  if constexpr (!TC) {
+    for (int l = 0; l < D.Le; ++l) {
+      const EncLayerW<W>& L = mw.enc[l];
+      prefetch_gemm_weights(L.wqkv, 3 * D.d, D.d);
+      prefetch_gemm_weights(L.wo, D.d, D.d);
+      prefetch_gemm_weights(L.w1, D.f, D.d);
+      prefetch_gemm_weights(L.w2, D.d, D.f);
+    }
+    for (int l = 0; l < D.Ld; ++l) prefetch_gemm_weights(mw.dec[l].wkvc, 2 * D.d, D.d);
   }
-  for (int l = 0; l < D.Ld; ++l) prefetch_gemm_weights(mw.dec[l].wkvc, 2 * D.d, D.d);
-  auto barrier = [&] { return grid_barrier(B.bar, tgt, status, [&] { stream_weights(P, smem); }); };
+  auto barrier = [&] { return grid_barrier(B.bar, tgt, status, [&] { stream_weights<W, TC>(P, smem); }); };
 
   for (int l = 0; l < D.Le; ++l) {
     const EncLayerW<W>& L = mw.enc[l];
@@ -784,7 +809,7 @@ __device__ bool encode_pass(const KParams<W>& P, unsigned char* smem, unsigned& 
     g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
     g.kdst_f = B.k; g.vdst_f = B.v;
     gemm_plan(g, gridDim.x);
-    if (!run_gemm<W>(P, g, T, 4 * l + TE_QKV, smem) || !barrier()) return false;
+    if (!run_gemm<W, TC>(P, g, T, 4 * l + TE_QKV, smem) || !barrier()) return false;
 
     attn_phase<float, W>(D, B.q, B.k, B.v, B.att, n, nullptr, nullptr, n, scratch);
     if (!barrier()) return false;
@@ -793,7 +818,7 @@ __device__ bool encode_pass(const KParams<W>& P, unsigned char* smem, unsigned& 
     g.M = n; g.N = D.d; g.K = D.d; g.xw_src = B.att; g.w = L.wo; g.bias = L.bo;
     g.epi = EPI_RESID; g.out = B.rb; g.ld = D.d; g.resid = res1;
     gemm_plan(g, gridDim.x);
-    if (!run_gemm<W>(P, g, T, 4 * l + TE_O, smem) || !barrier()) return false;
+    if (!run_gemm<W, TC>(P, g, T, 4 * l + TE_O, smem) || !barrier()) return false;
 
     g = GemmArgs<W>{};
     g.M = n; g.N = D.f; g.K = D.d; g.x_src = B.rb;
@@ -802,16 +827,17 @@ __device__ bool encode_pass(const KParams<W>& P, unsigned char* smem, unsigned& 
     const float* res2 = pre ? B.rb : B.xb;
     g.w = L.w1; g.bias = L.b1; g.epi = EPI_ACT; g.out_w = B.ffh; g.ld = D.f;
     gemm_plan(g, gridDim.x);
-    if (!run_gemm<W>(P, g, T, 4 * l + TE_FFN1, smem) || !barrier()) return false;
+    if (!run_gemm<W, TC>(P, g, T, 4 * l + TE_FFN1, smem) || !barrier()) return false;
 
     g = GemmArgs<W>{};
     g.M = n; g.N = D.d; g.K = D.f; g.xw_src = B.ffh; g.w = L.w2; g.bias = L.b2;
     g.epi = EPI_RESID; g.out = B.ra; g.ld = D.d; g.resid = res2;
     gemm_plan(g, gridDim.x);
-    if (!run_gemm<W>(P, g, T, 4 * l + TE_FFN2, smem) || !barrier()) return false;
+    if (!run_gemm<W, TC>(P, g, T, 4 * l + TE_FFN2, smem) || !barrier()) return false;
   }
   // cross-attention keys and values of every decoder layer from the encoder output, into the
-  // sentence's slot (independent phases: no barrier between them)
+  // sentence's slot (independent phases: no barrier between them, unless their K is split,
+  // whose partial sums and arrival counters the next phase reuses)
   const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
   const size_t slot_off = (size_t)P.enc_slot * D.max_src * D.d;
   for (int l = 0; l < D.Ld; ++l) {
@@ -823,20 +849,24 @@ __device__ bool encode_pass(const KParams<W>& P, unsigned char* smem, unsigned& 
     g.kdst = B.kcross + l * cross_ld + slot_off;
     g.vdst = B.vcross + l * cross_ld + slot_off;
     gemm_plan(g, gridDim.x);
-    if (!run_gemm<W>(P, g, T, 4 * D.Le + l, smem)) return false;
+    if (!run_gemm<W, TC>(P, g, T, 4 * D.Le + l, smem)) return false;
+    if constexpr (TC) {
+      if (l + 1 < D.Ld && gemm_geom(D, TC_ENCODE, 4 * D.Le + l).S > 1 && !barrier()) return false;
+    }
   }
   return true;
 }
 
-template <typename W>
-__global__ void __launch_bounds__(kThreads, 1) encode_kernel(KParams<W> P) {
+template <typename W, bool TC>
+__global__ void __launch_bounds__(kThreads, 1) encode_kernel(const __grid_constant__ KParams<W> P) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   unsigned char* smem = smem_base<W>(smem_raw);
   unsigned tgt = 0;
   load_smem_mw(P);
-  if constexpr (kTensorCores<W>) tc_setup<W>(P.D, TC_ENCODE, smem_layout(P.D, sizeof(W)).ring_slots);
-  (void)encode_pass<W>(P, smem, tgt);
-  if constexpr (kTensorCores<W>) tc_teardown<W>();
+  const Dims& D = smem_dims<W>();
+  if constexpr (TC) tc_setup<W>(D, TC_ENCODE, smem_layout(D, sizeof(W)).ring_slots, P.maps);
+  (void)encode_pass<W, TC>(P, smem, tgt);
+  if constexpr (TC) tc_teardown<W>();
 }
 
 }  // namespace pd
@@ -868,6 +898,7 @@ struct pd_ctx {
   int n_encoded = 0;                          // slots 0..n_encoded-1 hold encoded sentences
   int64_t launches = 0;
   float* static_logits = nullptr;              // device address of the fixed logits array
+  std::vector<CUtensorMap> dec_maps, enc_maps; // bf16: per GEMM phase of each kernel
   std::string err;
 };
 
@@ -908,6 +939,7 @@ bool valid_config(const pd_config* c, std::string* why) {
     if (id < 0 || id >= c->vocab) return bad("special ids must be in [0, vocab)");
   if (!(c->ln_eps >= 0.f)) return bad("ln_eps");
   if (c->max_batch < 0 || c->max_batch > pd::kMaxBatch) return bad("max_batch must be in [0, 64]");
+  if (c->gemm_engine < PD_ENGINE_AUTO || c->gemm_engine > PD_ENGINE_TENSOR) return bad("gemm_engine");
   if (c->dtype == PD_DTYPE_BF16 && c->vocab < pd::kTileN)
     return bad("bf16 models need vocab >= 128 (one tensor-core tile)");
   return true;
@@ -979,6 +1011,16 @@ pd_status dalloc(pd_ctx* c, T** p, size_t count) {
     if (s_ != PD_OK) return s_;    \
   } while (0)
 
+// The decode / encode kernel of a context's engine (bf16 only has the tensor-core one).
+template <typename W>
+const void* kernel_fn(bool encode, bool tc) {
+  if constexpr (sizeof(W) == 2) {
+    if (tc) return encode ? (const void*)pd::encode_kernel<W, true>
+                          : (const void*)pd::decode_kernel<W, true>;
+  }
+  return encode ? (const void*)pd::encode_kernel<W, false> : (const void*)pd::decode_kernel<W, false>;
+}
+
 pd_status raise_smem_limit(pd_ctx* c, const void* fn) {
   cudaFuncAttributes a{};
   PD_CUDA(c, cudaFuncGetAttributes(&a, fn));
@@ -1011,45 +1053,46 @@ pd_status tc_resources(pd_ctx* c, const pd::ModelW<__nv_bfloat16>& mw) {
   const Dims& D = c->D;
   PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
   if (!enc) return fail(c, PD_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
-  std::vector<CUtensorMap> maps(pd::kNumTmaps);
-  std::memset(maps.data(), 0, maps.size() * sizeof(CUtensorMap));
-  auto make = [&](int idx, const __nv_bfloat16* w, int N, int K) -> pd_status {
+  auto make = [&](CUtensorMap* m, const __nv_bfloat16* w, int N, int K) -> pd_status {
+    std::memset(m, 0, sizeof(CUtensorMap));
     cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)N};
     cuuint64_t strides[1] = {(cuuint64_t)K * 2};
     cuuint32_t box[2] = {(cuuint32_t)pd::kKBlock, (cuuint32_t)pd::kTileN};
     cuuint32_t estr[2] = {1, 1};
-    const CUresult r = enc(&maps[idx], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                           const_cast<__nv_bfloat16*>(w), dims, strides, box, estr,
-                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<__nv_bfloat16*>(w),
+                           dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS)
       return fail(c, PD_ECUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
     return PD_OK;
   };
-  const int d = D.d, f = D.f;
-  for (int l = 0; l < D.Le; ++l) {
-    const auto& L = mw.enc[l];
-    PD_TRY(make(4 * l + 0, L.wqkv, 3 * d, d));
-    PD_TRY(make(4 * l + 1, L.wo, d, d));
-    PD_TRY(make(4 * l + 2, L.w1, f, d));
-    PD_TRY(make(4 * l + 3, L.w2, d, f));
+  // the weight matrix of GEMM phase g of each kernel's phase sequence (pd::gemm_geom order)
+  for (int kind : {pd::TC_DECODE, pd::TC_ENCODE}) {
+    std::vector<CUtensorMap>& maps = kind == pd::TC_DECODE ? c->dec_maps : c->enc_maps;
+    const int n = pd::gemm_phase_count(D, kind);
+    maps.assign(n, CUtensorMap{});
+    for (int g = 0; g < n; ++g) {
+      const pd::Geom G = pd::gemm_geom(D, kind, g);
+      const __nv_bfloat16* w;
+      if (kind == pd::TC_DECODE) {
+        if (g == 6 * D.Ld) {
+          w = mw.embed;
+        } else {
+          const auto& L = mw.dec[g / 6];
+          const __nv_bfloat16* t[6] = {L.wqkv, L.wo, L.wqc, L.woc, L.w1, L.w2};
+          w = t[g % 6];
+        }
+      } else if (g >= 4 * D.Le) {
+        w = mw.dec[g - 4 * D.Le].wkvc;
+      } else {
+        const auto& L = mw.enc[g / 4];
+        const __nv_bfloat16* t[4] = {L.wqkv, L.wo, L.w1, L.w2};
+        w = t[g % 4];
+      }
+      PD_TRY(make(&maps[g], w, G.N, G.K));
+    }
   }
-  for (int l = 0; l < D.Ld; ++l) {
-    const auto& L = mw.dec[l];
-    const int b = pd::kTmapDec + 7 * l;
-    PD_TRY(make(b + 0, L.wqkv, 3 * d, d));
-    PD_TRY(make(b + 1, L.wo, d, d));
-    PD_TRY(make(b + 2, L.wqc, d, d));
-    PD_TRY(make(b + 3, L.woc, d, d));
-    PD_TRY(make(b + 4, L.w1, f, d));
-    PD_TRY(make(b + 5, L.w2, d, f));
-    PD_TRY(make(b + 6, L.wkvc, 2 * d, d));
-  }
-  PD_TRY(make(pd::kTmapEmbed, mw.embed, D.V, d));
-  CUtensorMap* dmaps = nullptr;
-  PD_TRY(dalloc(c, &dmaps, maps.size()));
-  PD_CUDA(c, cudaMemcpy(dmaps, maps.data(), maps.size() * sizeof(CUtensorMap),
-                        cudaMemcpyHostToDevice));
   // the largest split-K partial buffer any GEMM phase needs: S x N x rows floats
   size_t red = 1;
   for (int kind : {pd::TC_DECODE, pd::TC_ENCODE})
@@ -1058,13 +1101,11 @@ pd_status tc_resources(pd_ctx* c, const pd::ModelW<__nv_bfloat16>& mw) {
       if (G.S > 1) red = std::max(red, (size_t)G.S * G.N * D.rows);
     }
   pd::Bufs<__nv_bfloat16>& B = c->bb;
-  B.tmaps = dmaps;
   PD_TRY(dalloc(c, &B.red, red));
   PD_TRY(dalloc(c, &B.cnt, (size_t)pd::kCounterSlots));
   PD_CUDA(c, cudaMemset(B.cnt, 0, pd::kCounterSlots * sizeof(unsigned)));
   return PD_OK;
 }
-pd_status tc_resources(pd_ctx*, const pd::ModelW<float>&) { return PD_OK; }
 
 template <typename W>
 pd_status create_impl(pd_ctx* c, const void* weights) {
@@ -1126,20 +1167,22 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
   PD_CUDA(c, cudaMemset(B.st, 0, sizeof(pd::DecState)));
   PD_CUDA(c, cudaMemset(B.bar, 0, 4 * sizeof(unsigned)));
 
-  if constexpr (sizeof(W) == 2) PD_TRY(tc_resources(c, mw));
+  if constexpr (sizeof(W) == 2) {
+    if (D.tc) PD_TRY(tc_resources(c, mw));
+  }
 
   c->smem = pd::smem_layout(D, sizeof(W)).total;
-  if (sizeof(W) == 2 && pd::smem_layout(D, sizeof(W)).ring_slots < 2)
+  if (D.tc && pd::smem_layout(D, sizeof(W)).ring_slots < 2)
     return fail(c, PD_EINVAL, "the tensor-core kernels' shared memory does not fit (max_tgt_len "
                               "or max_batch too large)");
   // the limit is per kernel function and shared by every context of the process: only raise it
-  PD_TRY(raise_smem_limit(c, (const void*)pd::decode_kernel<W>));
-  PD_TRY(raise_smem_limit(c, (const void*)pd::encode_kernel<W>));
+  const void* fdec = kernel_fn<W>(false, D.tc != 0);
+  const void* fenc = kernel_fn<W>(true, D.tc != 0);
+  PD_TRY(raise_smem_limit(c, fdec));
+  PD_TRY(raise_smem_limit(c, fenc));
   int nb1 = 0, nb2 = 0;
-  PD_CUDA(c, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb1, pd::decode_kernel<W>, pd::kThreads,
-                                                           c->smem));
-  PD_CUDA(c, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb2, pd::encode_kernel<W>, pd::kThreads,
-                                                           c->smem));
+  PD_CUDA(c, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb1, fdec, pd::kThreads, c->smem));
+  PD_CUDA(c, cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb2, fenc, pd::kThreads, c->smem));
   if (nb1 < 1 || nb2 < 1) return fail(c, PD_EINVAL, "kernel does not fit on an SM (shared memory)");
   return PD_OK;
 }
@@ -1161,8 +1204,12 @@ pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P, bool reset_status = 
   PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).bar, 0, 4 * sizeof(unsigned), c->stream));
   if (encode && reset_status)
     PD_CUDA(c, cudaMemsetAsync(bufs<W>(c).st, 0, sizeof(pd::DecState), c->stream));
+  if (c->D.tc) {                              // the kernel's tensor maps ride in its parameters
+    const std::vector<CUtensorMap>& maps = encode ? c->enc_maps : c->dec_maps;
+    std::memcpy(P.maps, maps.data(), maps.size() * sizeof(CUtensorMap));
+  }
   void* args[] = {&P};
-  const void* fn = encode ? (const void*)pd::encode_kernel<W> : (const void*)pd::decode_kernel<W>;
+  const void* fn = kernel_fn<W>(encode, c->D.tc != 0);
   PD_CUDA(c, cudaLaunchCooperativeKernel(fn, dim3(c->grid), dim3(pd::kThreads), args, c->smem,
                                          c->stream));
   c->launches += 1;
@@ -1293,6 +1340,9 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   D.max_batch = cfg->max_batch > 1 ? cfg->max_batch : 1;
   const long batch_rows = std::min<long>((long)D.max_batch * D.max_tgt, pd::kMaxPassRows);
   D.rows = (int)std::max<long>(D.max_keys, batch_rows);
+  D.tc = cfg->dtype == PD_DTYPE_BF16 &&
+         (cfg->gemm_engine == PD_ENGINE_TENSOR ||
+          (cfg->gemm_engine == PD_ENGINE_AUTO && D.max_batch > 1));
   c->blob_bytes = nbytes;
   pd_status s = PD_OK;
   cudaError_t e = cudaGetDevice(&c->device);

@@ -67,6 +67,7 @@ struct Dims {
   int max_keys;    // max(max_src, max_tgt): rows of the position table, keys of an attention row
   int max_batch;   // sentences one decode carries (cache slots per layer)
   int rows;        // activation rows: max(max_keys, min(max_batch * max_tgt, kMaxPassRows))
+  int tc;          // bf16: GEMM phases on the tensor cores (else the SIMT path)
 };
 
 // Per-CTA partial of the LM-head argmax for one row.
@@ -108,7 +109,6 @@ struct Bufs {
   int* src;                    // [max_src]
   int* dbg_tok;                // [max_tgt]
   float* pos_tab;              // sinusoidal positions [rows][d] (built once at create)
-  const void* tmaps;           // bf16: CUtensorMap of every weight matrix (device memory)
   float* red;                  // bf16: split-K partial sums [S][rows][N]
   unsigned* cnt;               // bf16: split-K arrival counters (zero between uses)
 };

@@ -37,12 +37,13 @@ constexpr int kTileN = 128;            // output features per tile (the MMA's M)
 constexpr int kKBlock = 64;            // K elements of one TMA box (128 bytes of bf16)
 constexpr int kSlotBytes = kTileN * kKBlock * 2;
 constexpr int kRowTile = 16;           // token rows per MMA (the MMA's N)
-constexpr int kBBytes = 32 * 1024;     // staged token rows (B operand)
+constexpr int kBBytes = 64 * 1024;     // staged token rows (B operand)
 constexpr int kKSliceMax = 512;        // K per item of a split phase
-constexpr int kMaxChunk = 32;          // token rows per chunk (B buffer and TMEM columns)
+constexpr int kMaxChunk = 128;         // token rows per chunk (B buffer, MMA N, TMEM columns)
 constexpr int kEpiLd = kTileN + 4;     // floats per row of the epilogue tile
 constexpr int kEpiBytes = kRowTile * kEpiLd * 4;
-constexpr int kTmemCols = 64;
+constexpr int kAccs = 4;               // independent accumulators per item (K-block kb -> kb % 4)
+constexpr int kTmemCols = kAccs * kMaxChunk;
 constexpr int kMaxGemmPhases = 8 * kMaxLayers + 1;
 constexpr int kCounterSlots = 8192;    // split-K arrival counters (tile x chunk)
 
@@ -55,18 +56,26 @@ enum : int { TD_QKV = 0, TD_O = 1, TD_QC = 2, TD_OC = 3, TD_FFN1 = 4, TD_FFN2 = 
 // projection of decoder layer l).
 enum : int { TE_QKV = 0, TE_O = 1, TE_FFN1 = 2, TE_FFN2 = 3 };
 
-// Tensor maps of the weight matrices (one CUtensorMap each, in device memory): encoder layer l
-// at 4 l + {wqkv, wo, w1, w2}; decoder layer l at kTmapDec + 7 l + {wqkv, wo, wqc, woc, w1, w2,
-// wkvc}; the (tied) embedding last.
-constexpr int kTmapDec = 4 * kMaxLayers;
-constexpr int kTmapEmbed = kTmapDec + 7 * kMaxLayers;
-constexpr int kNumTmaps = kTmapEmbed + 1;
+// Each kernel receives, among its parameters, one TMA tensor map per GEMM phase of its phase
+// sequence (index = the phase's GEMM index g): parameter space is read through the constant
+// cache, so issuing a TMA load does not wait for a descriptor fetch from device memory.
+constexpr int kMaxKernelMaps = 6 * kMaxLayers + 1;
 
 struct Geom {
-  int tmap;          // index into the tensor-map array
+  int tmap;          // index of the phase's tensor map among the kernel's parameters
   int N, K, S, KS;   // outputs, inputs, K split, K per item
   int RC;            // token rows per chunk
   int tiles, items;
+};
+
+// One GEMM phase as this CTA sees it (computed once per kernel, in shared memory, so that the
+// single thread driving the weight stream and the MMAs does no division on its critical path):
+// N outputs, items = tiles x S, this CTA's items first, first + grid, ... (nj of them), S K-slices
+// of kbs K-blocks, token rows per chunk 1 << rc_sh.
+struct PInfo {
+  int N, items;
+  short first, nj;
+  unsigned char S, kbs, rc_sh, pad;
 };
 
 // Per-CTA state of the tensor-core path (shared memory).  Only thread 0 touches the stream
@@ -76,9 +85,9 @@ struct TcState {
   unsigned long long empty[kRingMax];  // slot read by its MMAs (tcgen05.commit)
   unsigned long long acc;              // an item's MMAs are done (tcgen05.commit)
   uint32_t tmem;                       // tensor-memory base address
-  int ring;                            // slots in use
+  int ring, ring_sh;                   // slots in use (a power of two) and its log2
   int kind, n_g;                       // phase sequence and its GEMM phase count
-  int off[kMaxGemmPhases];             // rotation offset of each GEMM phase
+  PInfo info[kMaxGemmPhases];          // the kernel's GEMM phases as this CTA sees them
   // weight stream cursor: phase, chunk, item of this CTA, K-block; sequence number
   int p_g, p_chunk, p_j, p_kb, p_seq, p_M, p_open;
   int c_seq;                           // K-blocks consumed
@@ -258,62 +267,78 @@ __host__ __device__ inline int gemm_phase_count(const Dims& D, int kind) {
 __host__ __device__ inline Geom gemm_geom(const Dims& D, int kind, int g) {
   const int d = D.d, f = D.f;
   if (kind == TC_DECODE) {
-    if (g == 6 * D.Ld) return make_geom(kTmapEmbed, D.V, d, true);
-    const int l = g / 6, t = g % 6, base = kTmapDec + 7 * l;
-    switch (t) {
-      case TD_QKV: return make_geom(base + 0, 3 * d, d, false);
-      case TD_O: return make_geom(base + 1, d, d, false);
-      case TD_QC: return make_geom(base + 2, d, d, false);
-      case TD_OC: return make_geom(base + 3, d, d, false);
-      case TD_FFN1: return make_geom(base + 4, f, d, false);
-      default: return make_geom(base + 5, d, f, false);
+    if (g == 6 * D.Ld) return make_geom(g, D.V, d, true);
+    switch (g % 6) {
+      case TD_QKV: return make_geom(g, 3 * d, d, false);
+      case TD_O: return make_geom(g, d, d, false);
+      case TD_QC: return make_geom(g, d, d, false);
+      case TD_OC: return make_geom(g, d, d, false);
+      case TD_FFN1: return make_geom(g, f, d, false);
+      default: return make_geom(g, d, f, false);
     }
   }
-  if (g >= 4 * D.Le) return make_geom(kTmapDec + 7 * (g - 4 * D.Le) + 6, 2 * d, d, false);
-  const int l = g / 4, t = g % 4, base = 4 * l;
-  switch (t) {
-    case TE_QKV: return make_geom(base + 0, 3 * d, d, false);
-    case TE_O: return make_geom(base + 1, d, d, false);
-    case TE_FFN1: return make_geom(base + 2, f, d, false);
-    default: return make_geom(base + 3, d, f, false);
+  if (g >= 4 * D.Le) return make_geom(g, 2 * d, d, false);
+  switch (g % 4) {
+    case TE_QKV: return make_geom(g, 3 * d, d, false);
+    case TE_O: return make_geom(g, d, d, false);
+    case TE_FFN1: return make_geom(g, f, d, false);
+    default: return make_geom(g, d, f, false);
   }
-}
-
-// Item j of this CTA in a phase with rotation offset off (-1: none left).
-__device__ __forceinline__ int cta_item(const Geom& G, int off, int j) {
-  const int grid = (int)gridDim.x;
-  const int first = ((int)blockIdx.x - off % grid + grid) % grid;
-  const int i = first + j * grid;
-  return i < G.items ? i : -1;
-}
-__device__ __forceinline__ int cta_items(const Geom& G, int off) {
-  const int grid = (int)gridDim.x;
-  const int first = ((int)blockIdx.x - off % grid + grid) % grid;
-  return first < G.items ? (G.items - first + grid - 1) / grid : 0;
 }
 
 // ------------------------------------------------------------------------------------------
 // set-up, weight stream, tear-down
 // ------------------------------------------------------------------------------------------
 
-// Every thread.  ring = slots that fit; kind = the phase sequence this kernel runs.
+// Every thread.  ring = slots that fit; kind = the phase sequence this kernel runs; maps = its
+// tensor maps (kernel parameters).
 template <typename W>
-__device__ void tc_setup(const Dims& D, int kind, int ring) {
+__device__ void tc_setup(const Dims& D, int kind, int ring, const CUtensorMap* maps) {
   TcState& s = smem_tc<W>();
+  for (int g = threadIdx.x; g < gemm_phase_count(D, kind); g += kThreads)
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(maps + g)) : "memory");
+  const int n_g = gemm_phase_count(D, kind);
+  const int grid = (int)gridDim.x;
+  for (int g = threadIdx.x; g < n_g; g += kThreads) {        // one phase per thread
+    const Geom G = gemm_geom(D, kind, g);
+    PInfo& in = s.info[g];
+    in.N = G.N;
+    in.items = G.items;
+    in.S = (unsigned char)G.S;
+    in.kbs = (unsigned char)(G.KS / kKBlock);
+    int sh = 4;
+    while ((2 << sh) <= G.RC) ++sh;
+    in.rc_sh = (unsigned char)sh;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {          // rotation: phase g starts at CTA (items of phases < g) % grid
+    int off = 0;
+    for (int g = 0; g < n_g; ++g) {
+      s.info[g].first = (short)off;           // the offset, for now
+      off += s.info[g].items;
+      while (off >= grid) off -= grid;
+    }
+  }
+  __syncthreads();
+  for (int g = threadIdx.x; g < n_g; g += kThreads) {
+    PInfo& in = s.info[g];
+    int first = (int)blockIdx.x - in.first;
+    if (first < 0) first += grid;
+    in.first = (short)first;
+    in.nj = (short)(first < in.items ? (in.items - first + grid - 1) / grid : 0);
+  }
   if (threadIdx.x == 0) {
-    for (int i = 0; i < ring; ++i) {
+    for (int i = 0; i < kRingMax; ++i) {
       mbar_init(&s.full[i], 1);
       mbar_init(&s.empty[i], 1);
     }
     mbar_init(&s.acc, 1);
-    s.ring = ring;
+    int sh = 0;
+    while ((2 << sh) <= ring) ++sh;
+    s.ring = 1 << sh;
+    s.ring_sh = sh;
     s.kind = kind;
-    s.n_g = gemm_phase_count(D, kind);
-    int off = 0;
-    for (int g = 0; g < s.n_g; ++g) {
-      s.off[g] = off;
-      off = (off + gemm_geom(D, kind, g).items) % (int)gridDim.x;
-    }
+    s.n_g = n_g;
     s.p_g = 0; s.p_chunk = 0; s.p_j = 0; s.p_kb = 0; s.p_seq = 0; s.p_M = 0; s.p_open = 0;
     s.c_seq = 0; s.acc_n = 0; s.last = 0; s.err = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -334,42 +359,50 @@ template <typename W>
 __device__ void tc_produce(const Dims& D, const CUtensorMap* maps, unsigned char* ring,
                            bool block) {
   TcState& s = smem_tc<W>();
-  while (s.p_g < s.n_g) {
-    const Geom G = gemm_geom(D, s.kind, s.p_g);
-    const int nj = cta_items(G, s.off[s.p_g]);
-    const int M = s.p_M;
-    const int nch = M > 0 ? (M + G.RC - 1) / G.RC : 1;
-    if (nj == 0 || s.p_chunk >= nch) {          // next phase
+  // the cursor in registers (the asm statements below clobber memory, which would make the
+  // compiler reload every shared field after each of them)
+  int g = s.p_g, chunk = s.p_chunk, j = s.p_j, kb = s.p_kb, seq = s.p_seq, M = s.p_M;
+  int open = s.p_open;
+  const int n_g = s.n_g, rsh = s.ring_sh, rmask = (1 << rsh) - 1;
+  const int grid = (int)gridDim.x;
+  PInfo in = g < n_g ? s.info[g] : PInfo{};
+  int nch = M > 0 ? (M + (1 << in.rc_sh) - 1) >> in.rc_sh : 1;
+  while (g < n_g) {
+    if (in.nj == 0 || chunk >= nch) {            // next phase
       // between passes the row count is unknown: past the first chunk of the first phase
       // with items, the order of the blocks depends on it
-      if (M == 0 && nj > 0) return;
-      s.p_g += 1; s.p_chunk = 0; s.p_j = 0; s.p_kb = 0;
-      if (s.p_g >= s.n_g) {
-        if (s.p_open) { s.p_g = 0; s.p_M = 0; s.p_open = 0; }   // wrap to the next pass
-        else return;
+      if (M == 0 && in.nj > 0) break;
+      g += 1; chunk = 0; j = 0; kb = 0;
+      if (g >= n_g) {
+        if (!open) break;
+        g = 0; M = 0; open = 0;                  // wrap to the next pass
       }
+      in = s.info[g];
+      nch = M > 0 ? (M + (1 << in.rc_sh) - 1) >> in.rc_sh : 1;
       continue;
     }
-    const int slot = s.p_seq % s.ring, use = s.p_seq / s.ring;
+    const int slot = seq & rmask, use = seq >> rsh;
     if (use > 0) {
       if (block) {
-        if (!mbar_wait(&s.empty[slot], (use - 1) & 1, &s.err)) return;
+        if (!mbar_wait(&s.empty[slot], (use - 1) & 1, &s.err)) break;
       } else if (!mbar_test(&s.empty[slot], (use - 1) & 1)) {
-        return;
+        break;
       }
     }
-    const int i = cta_item(G, s.off[s.p_g], s.p_j);
-    const int tile = i / G.S, sp = i % G.S;
+    const int i = in.first + j * grid;
+    const int tile = in.S == 1 ? i : i / in.S, sp = in.S == 1 ? 0 : i - tile * in.S;
     mbar_expect_tx(&s.full[slot], kSlotBytes);
-    tma_load_2d(ring + (size_t)slot * kSlotBytes, maps + G.tmap, &s.full[slot],
-                sp * G.KS + s.p_kb * kKBlock, tile * kTileN);
-    s.p_seq += 1;
-    if (++s.p_kb == G.KS / kKBlock) {
-      s.p_kb = 0;
-      if (++s.p_j == nj) { s.p_j = 0; s.p_chunk += 1; }
+    tma_load_2d(ring + (size_t)slot * kSlotBytes, maps + g, &s.full[slot],
+                (sp * in.kbs + kb) * kKBlock, tile * kTileN);
+    seq += 1;
+    if (++kb == in.kbs) {
+      kb = 0;
+      if (++j == in.nj) { j = 0; chunk += 1; }
     }
-    if (block) return;
+    if (block) break;
   }
+  s.p_g = g; s.p_chunk = chunk; s.p_j = j; s.p_kb = kb; s.p_seq = seq; s.p_M = M;
+  s.p_open = open;
 }
 
 // Thread 0, at the start of a pass of M rows (pass_open: keep streaming into the next pass).
@@ -388,7 +421,7 @@ __device__ void tc_teardown() {
   __syncthreads();
   if (threadIdx.x == 0) {
     for (int q = s.c_seq; q < s.p_seq; ++q)
-      (void)mbar_wait(&s.full[q % s.ring], (q / s.ring) & 1, &s.err, 1000000000ull);
+      (void)mbar_wait(&s.full[q & (s.ring - 1)], (q >> s.ring_sh) & 1, &s.err, 1000000000ull);
     mma_commit(&s.acc);
     (void)mbar_wait(&s.acc, s.acc_n & 1, &s.err, 1000000000ull);
   }
@@ -544,6 +577,53 @@ __device__ __forceinline__ void epi_store(const GemmArgs<W>& g, const Dims& D, i
 
 constexpr int kArgRows = (kMaxChunk + kWarps - 1) / kWarps;   // chunk rows per warp (argmax)
 
+// Thread 0: the MMAs of one item over rtiles 16-row tiles.  K-block kb accumulates into
+// accumulator kb % kAccs (tensor-memory columns (kb % kAccs) * kMaxChunk + 16 rt ..), so that
+// kAccs dependent chains of MMAs run side by side; within a chain the K-blocks and the K = 16
+// steps are in ascending order.  Every K-block's slot is released by a commit once its MMAs
+// are done.  Returns false if the weight stream or a wait failed.
+template <typename W>
+__device__ __forceinline__ bool tc_issue_item(const Dims& D, const CUtensorMap* maps,
+                                              unsigned char* ring, unsigned char* bb, int kbs,
+                                              int rtiles) {
+  TcState& s = smem_tc<W>();
+  const uint32_t idesc = idesc_bf16(kTileN, kRowTile * rtiles);
+  const uint32_t bbase = smem_u32(bb);
+  const uint32_t tmem = s.tmem;
+  const int rmask = s.ring - 1, rsh = s.ring_sh;
+  const uint32_t rbase = smem_u32(ring);
+  int cseq = s.c_seq;
+  bool ok = true;
+  tc_fence_after();
+  for (int kb = 0; kb < kbs && ok; ++kb) {
+    while (s.p_seq <= cseq) {
+      const int before = s.p_seq;
+      tc_produce<W>(D, maps, ring, true);
+      if (s.err) { ok = false; break; }
+      if (s.p_seq == before) { s.err = 2; ok = false; break; }   // the stream cannot supply it
+    }
+    if (!ok) break;
+    const int slot = cseq & rmask, use = cseq >> rsh;
+    if (!mbar_wait(&s.full[slot], use & 1, &s.err)) { ok = false; break; }
+    tc_fence_after();
+    // descriptors advance by 32 bytes (2 in the start-address field) per K = 16 step
+    const uint64_t a0 = sw128_desc(rbase + (uint32_t)(slot * kSlotBytes));
+    const uint32_t col = (uint32_t)((kb % kAccs) * kMaxChunk);
+    // one MMA covers every 16-row tile of the chunk (N = 16 rtiles): the B rows of a K-block
+    // are contiguous, 128 bytes apart, and the accumulator columns of the tiles adjacent
+    const uint64_t b0 = sw128_desc(bbase + (uint32_t)(kb * rtiles * 2048));
+#pragma unroll
+    for (int k16 = 0; k16 < kKBlock / 16; ++k16)
+      mma_bf16(tmem + col, a0 + (uint64_t)(2 * k16), b0 + (uint64_t)(2 * k16), idesc,
+               (kb >= kAccs || k16 > 0) ? 1u : 0u);
+    mma_commit(&s.empty[slot]);
+    cseq += 1;
+    tc_produce<W>(D, maps, ring, false);
+  }
+  s.c_seq = cseq;
+  return ok;
+}
+
 // GEMM phase g of the current phase sequence over the M rows of ga, on the tensor cores.
 // Every thread of every CTA calls it (CTAs without items of the phase only keep the weight
 // stream going and, for the LM head, publish empty argmax partials).  Returns false if a
@@ -554,15 +634,15 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
                                            unsigned char* ring, unsigned char* bb, float* epi,
                                            float* red, unsigned* cnt) {
   TcState& s = smem_tc<W>();
-  const Geom G = gemm_geom(D, s.kind, gph);
-  const int off = s.off[gph];
-  const int nj = cta_items(G, off);
+  const PInfo in = s.info[gph];
+  const int nj = in.nj, S = in.S, kbs = in.kbs, KS = kbs * kKBlock, N = in.N;
+  const int RC = 1 << in.rc_sh;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int M = ga.M;
-  const int nch = (M + G.RC - 1) / G.RC;
+  const int nch = (M + RC - 1) >> in.rc_sh;
   const bool argmax = ga.epi == EPI_ARGMAX;
-  const bool storer = cta_item(G, off, 0) == 0;      // the CTA holding item 0 stores x rows
-  const uint32_t idesc = idesc_bf16(kTileN, kRowTile);
+  const bool storer = in.first == 0;                 // the CTA holding item 0 stores x rows
+  const int naccs = kbs < kAccs ? kbs : kAccs;
   if (nj == 0) {
     if (argmax)
       for (int m = threadIdx.x; m < M; m += kThreads)
@@ -572,52 +652,30 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
   }
   int staged_key = -1;
   for (int ch = 0; ch < nch; ++ch) {
-    const int m0 = ch * G.RC, mt = M - m0 < G.RC ? M - m0 : G.RC;
+    const int m0 = ch * RC, mt = M - m0 < RC ? M - m0 : RC;
     const int rtiles = (mt + kRowTile - 1) / kRowTile;
     Partial ap[kArgRows];
 #pragma unroll
     for (int k = 0; k < kArgRows; ++k) ap[k] = Partial{-INFINITY, 0x7fffffff, 0.f, 0};
     for (int j = 0; j < nj; ++j) {
-      const int i = cta_item(G, off, j);
-      const int tile = i / G.S, sp = i % G.S, n0 = tile * kTileN;
+      const int i = in.first + j * (int)gridDim.x;
+      const int tile = S == 1 ? i : i / S, sp = S == 1 ? 0 : i - tile * S;
+      const int n0 = tile * kTileN;
       // stage the B operand (rows of this chunk, the item's K-slice) when it changes
-      const int key = ch * G.S + sp;
+      const int key = ch * S + sp;
       if (key != staged_key) {
         __syncthreads();                           // the previous MMAs are done (acc wait)
-        stage_b<W>(ga, T, D, m0, mt, sp * G.KS, G.KS, rtiles, storer && sp == 0, bb);
+        stage_b<W>(ga, T, D, m0, mt, sp * KS, KS, rtiles, storer && sp == 0, bb);
         fence_proxy_async_smem();
         __syncthreads();
         staged_key = key;
       }
-      // per-thread epilogue operands that do not depend on this phase's products
+      // per-thread epilogue operand that does not depend on this phase's products
       const int f = threadIdx.x % kTileN;
       const int nf = n0 + f;
-      const float bias = (ga.bias != nullptr && nf < G.N) ? to_f(ga.bias[nf]) : 0.f;
-      // thread 0: the item's MMAs (K-blocks in ascending order, 16-row tiles, K = 16 steps)
+      const float bias = (ga.bias != nullptr && nf < N) ? to_f(ga.bias[nf]) : 0.f;
       if (threadIdx.x == 0) {
-        tc_fence_after();
-        for (int kb = 0; kb < G.KS / kKBlock && s.err == 0; ++kb) {
-          while (s.p_seq <= s.c_seq && s.err == 0) {
-            const int before = s.p_seq;
-            tc_produce<W>(D, maps, ring, true);
-            if (s.p_seq == before && s.err == 0) s.err = 2;    // the stream cannot supply it
-          }
-          if (s.err) break;
-          const int slot = s.c_seq % s.ring, use = s.c_seq / s.ring;
-          if (!mbar_wait(&s.full[slot], use & 1, &s.err)) break;
-          tc_fence_after();
-          const uint32_t a0 = smem_u32(ring + (size_t)slot * kSlotBytes);
-          const uint32_t b0 = smem_u32(bb) + (uint32_t)(kb * rtiles * 2048);
-          for (int rt = 0; rt < rtiles; ++rt)
-#pragma unroll
-            for (int k16 = 0; k16 < kKBlock / 16; ++k16)
-              mma_bf16(s.tmem + (uint32_t)(rt * kRowTile), sw128_desc(a0 + k16 * 32),
-                       sw128_desc(b0 + rt * 2048 + k16 * 32), idesc,
-                       (kb > 0 || k16 > 0) ? 1u : 0u);
-          mma_commit(&s.empty[slot]);
-          s.c_seq += 1;
-          tc_produce<W>(D, maps, ring, false);
-        }
+        (void)tc_issue_item<W>(D, maps, ring, bb, kbs, rtiles);
         mma_commit(&s.acc);
         (void)mbar_wait(&s.acc, s.acc_n & 1, &s.err);
       }
@@ -627,21 +685,28 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
       for (int rt = 0; rt < rtiles; ++rt) {
         const int rows = mt - rt * kRowTile < kRowTile ? mt - rt * kRowTile : kRowTile;
         if (warp < 4) {
-          float v[16];
-          tmem_ld16(s.tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(rt * kRowTile), v);
+          // the accumulators summed in a fixed order
+          const uint32_t ta = s.tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(rt * kRowTile);
+          float v[16], w[16];
+          tmem_ld16(ta, v);
+          for (int c = 1; c < naccs; ++c) {
+            tmem_ld16(ta + (uint32_t)(c * kMaxChunk), w);
+#pragma unroll
+            for (int r = 0; r < 16; ++r) v[r] += w[r];
+          }
 #pragma unroll
           for (int r = 0; r < 16; ++r) epi[r * kEpiLd + warp * 32 + lane] = v[r];
         }
         __syncthreads();
         bool mine = true;
-        if (G.S > 1) {
+        if (S > 1) {
           // split K: publish this slice's partial; the last of the S CTAs to arrive sums the
           // slices in ascending order and runs the epilogue
           const size_t rs = (size_t)D.rows;
           for (int e = threadIdx.x; e < rows * kTileN; e += kThreads) {
             const int r = e / kTileN, ff = e % kTileN, n = n0 + ff;
-            if (n < G.N)
-              red[((size_t)sp * rs + m0 + rt * kRowTile + r) * G.N + n] = epi[r * kEpiLd + ff];
+            if (n < N)
+              red[((size_t)sp * rs + m0 + rt * kRowTile + r) * N + n] = epi[r * kEpiLd + ff];
           }
           __threadfence();
           __syncthreads();
@@ -649,7 +714,7 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
             unsigned* c = cnt + (size_t)(tile * ((D.rows + kRowTile - 1) / kRowTile) +
                                          (m0 + rt * kRowTile) / kRowTile) % kCounterSlots;
             const unsigned old = atomicAdd(c, 1u);
-            s.last = old == (unsigned)(G.S - 1);
+            s.last = old == (unsigned)(S - 1);
             if (s.last) atomicExch(c, 0u);
           }
           __syncthreads();
@@ -659,9 +724,9 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
             for (int e = threadIdx.x; e < rows * kTileN; e += kThreads) {
               const int r = e / kTileN, ff = e % kTileN, n = n0 + ff;
               float acc = 0.f;
-              if (n < G.N)
-                for (int q = 0; q < G.S; ++q)
-                  acc += __ldcg(red + ((size_t)q * rs + m0 + rt * kRowTile + r) * G.N + n);
+              if (n < N)
+                for (int q = 0; q < S; ++q)
+                  acc += __ldcg(red + ((size_t)q * rs + m0 + rt * kRowTile + r) * N + n);
               epi[r * kEpiLd + ff] = acc;
             }
             __syncthreads();
@@ -679,20 +744,18 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                   const int ff = lane + 32 * q, n = n0 + ff;
-                  if (n < G.N)
+                  if (n < N)
                     argmax_push(epi[r * kEpiLd + ff], n, ap[k].mx, ap[k].idx, ap[k].sum,
                                 ap[k].nan);
                 }
               }
             }
-          } else {
+          } else if (nf < N) {
             // thread -> feature f = tid % 128 (one bias value), rows tid / 128 + 3 u
-            if (nf < G.N) {
-              for (int r = threadIdx.x / kTileN; r < rows; r += kThreads / kTileN) {
-                const int m = m0 + rt * kRowTile + r;
-                const float resid = ga.epi == EPI_RESID ? ga.resid[(size_t)m * ga.ld + nf] : 0.f;
-                epi_store<W>(ga, D, m, nf, epi[r * kEpiLd + f], bias, resid);
-              }
+            for (int r = threadIdx.x / kTileN; r < rows; r += kThreads / kTileN) {
+              const int m = m0 + rt * kRowTile + r;
+              const float resid = ga.epi == EPI_RESID ? ga.resid[(size_t)m * ga.ld + nf] : 0.f;
+              epi_store<W>(ga, D, m, nf, epi[r * kEpiLd + f], bias, resid);
             }
           }
         }

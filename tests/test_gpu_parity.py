@@ -50,14 +50,14 @@ def _gpu():
 
 
 class Setup:
-    def __init__(self, spec, max_src, max_tgt, eos=synth.EOS_ID, **wkw):
+    def __init__(self, spec, max_src, max_tgt, eos=synth.EOS_ID, engine="auto", **wkw):
         self.spec = spec
         self.eos = eos
         self.margin = MARGIN_BF16 if spec.dtype == synth.DTYPE_BF16 else MARGIN_F32
         self.w = synth.make_weights(spec, **wkw)
         self.model = om.Model(spec, self.w.tensors)
-        self.dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, eos_id=eos),
-                               self.w.blob)
+        self.dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, eos_id=eos,
+                                                    engine=engine), self.w.blob)
         self._mem = {}
 
     def mem(self, src):
@@ -139,16 +139,25 @@ BF16_KNOB = synth.small_spec("post-silu-bf16-knob", d_model=512, n_heads=8, d_ff
                              activation=synth.ACT_SILU, max_pos=128, dtype=synth.DTYPE_BF16)
 
 
-@pytest.fixture(scope="module")
-def bf16_knob():
-    s = Setup(BF16_KNOB, 64, 64, seed=12, ln_noise=1.0, embed_std=0.012)
+# bf16 models run with either matrix-product engine (pd_gemm_engine): the "_tc" fixtures use
+# the tensor cores (tcgen05), the others the SIMT path, each checked against the oracle.
+@pytest.fixture(scope="module", params=["simt", "tensor"])
+def bf16_knob(request):
+    s = Setup(BF16_KNOB, 64, 128, engine=request.param, seed=12, ln_noise=1.0, embed_std=0.012)
     yield s
     s.dec.close()
 
 
 @pytest.fixture(scope="module")
 def marian():
-    s = Setup(synth.MARIAN, 64, 128, seed=0)
+    s = Setup(synth.MARIAN, 64, 128, engine="simt", seed=0)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
+def marian_tc():
+    s = Setup(synth.MARIAN, 64, 128, engine="tensor", seed=0)
     yield s
     s.dec.close()
 
@@ -276,29 +285,31 @@ def test_tiny_logits_fp32(name, request):
         assert rel_row_err(got, ref).max() < 1e-4
 
 
-def test_marian_logits_bf16(marian):
+@pytest.mark.parametrize("name", ["marian", "marian_tc"])
+def test_marian_logits_bf16(name, request):
+    s = request.getfixturevalue(name)
     rng = np.random.default_rng(12)
-    for n_src, T in ((9, 12), (64, 40)):
-        src = rng.integers(3, marian.spec.vocab, size=n_src).astype(np.int32)
-        y_in = np.r_[synth.BOS_ID, rng.integers(3, marian.spec.vocab, size=T - 1)].astype(np.int32)
-        marian.dec.encode(src)
-        got = marian.dec.debug_logits(y_in)
-        ref = marian.model.logits(marian.mem(src), y_in)
+    for n_src, T in ((9, 12), (64, 40), (33, 128)):
+        src = rng.integers(3, s.spec.vocab, size=n_src).astype(np.int32)
+        y_in = np.r_[synth.BOS_ID, rng.integers(3, s.spec.vocab, size=T - 1)].astype(np.int32)
+        s.dec.encode(src)
+        got = s.dec.debug_logits(y_in)
+        ref = s.model.logits(s.mem(src), y_in)
         assert rel_row_err(got, ref).max() < 2e-2
 
 
-@pytest.mark.parametrize("name", ["tiny", "bf16_knob", "marian"])
+@pytest.mark.parametrize("name", ["tiny", "bf16_knob", "marian", "marian_tc"])
 def test_logits_batch_invariant(name, request):
     """Batch invariance, the property behind every method's bit identity with greedy: the
     logits of row t (inputs y_0..y_t) are the same bits whether the pass carries t + 1 rows or
-    more, whatever MMA tile, chunk or slot the row falls in (passes of 1 to 40 rows)."""
+    more, whatever MMA width, tile, chunk or slot the row falls in (passes of 1 to 128 rows)."""
     s = request.getfixturevalue(name)
     rng = np.random.default_rng(13)
     src = rng.integers(3, s.spec.vocab, size=19).astype(np.int32)
-    y_in = np.r_[synth.BOS_ID, rng.integers(3, s.spec.vocab, size=39)].astype(np.int32)
+    y_in = np.r_[synth.BOS_ID, rng.integers(3, s.spec.vocab, size=127)].astype(np.int32)
     s.dec.encode(src)
     full = s.dec.debug_logits(y_in)
-    for T in (1, 5, 16, 17, 33):
+    for T in (1, 5, 16, 17, 33, 64, 65, 100):
         part = s.dec.debug_logits(y_in[:T])
         assert np.array_equal(part.view(np.uint32), full[:T].view(np.uint32)), T
 
@@ -411,7 +422,7 @@ def test_bf16_traces_against_oracle(bf16_knob):
     assert early == 3
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_vary", "bf16_knob", "marian"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_vary", "bf16_knob", "marian", "marian_tc"])
 def test_trace_probs_against_own_logits_and_oracle(name, request):
     """The DDGviz probability of each greedy pass (softmax probability of the argmax, Section
     3.5) is computed on the device by an online sum of exponentials merged across CTA partials.
@@ -420,7 +431,7 @@ def test_trace_probs_against_own_logits_and_oracle(name, request):
     bound the measured logit error of each row gives: |d log p| <= 2 max_j |dl_j|."""
     s = request.getfixturevalue(name)
     for src in synth.sentences(23, 2, 6, 24, s.spec.vocab):
-        max_len = 2 * len(src) if name != "marian" else 12
+        max_len = 2 * len(src) if not name.startswith("marian") else 12
         s.dec.encode(src)
         g = s.dec.decode("greedy", max_len, trace=True)
         n = len(g.tokens)
@@ -439,7 +450,9 @@ def test_trace_probs_against_own_logits_and_oracle(name, request):
         assert (err <= 2 * dl + LOGP_SLACK).all(), err.max()
 
 
-def test_marian_methods_bit_identical(marian):
+@pytest.mark.parametrize("name", ["marian", "marian_tc"])
+def test_marian_methods_bit_identical(name, request):
+    marian = request.getfixturevalue(name)
     for src in synth.sentences(41, 3, 8, 12, marian.spec.vocab):
         max_len = 2 * len(src)
         marian.dec.encode(src)
@@ -453,9 +466,11 @@ def test_marian_methods_bit_identical(marian):
         assert frac >= MARIAN_MIN_COVERED
 
 
-def test_marian_full_size_sampled(marian):
+@pytest.mark.parametrize("name", ["marian", "marian_tc"])
+def test_marian_full_size_sampled(name, request):
     """The benchmark's launch configuration (GS-Jacobi b=5, max_len = 2n) on the longest
     sentence lengths of the workload: tokens checked by one teacher-forced oracle pass."""
+    marian = request.getfixturevalue(name)
     sents = synth.MARIAN_GS.sentences()
     longest = sorted(range(len(sents)), key=lambda k: -len(sents[k]))[:2]
     for k in longest:
@@ -595,9 +610,9 @@ def pre_f32():
     s.dec.close()
 
 
-@pytest.fixture(scope="module")
-def pre_bf16():
-    s = Setup(PRE_BF16, 64, 64, seed=12, ln_noise=0.2, embed_std=0.05)
+@pytest.fixture(scope="module", params=["simt", "tensor"])
+def pre_bf16(request):
+    s = Setup(PRE_BF16, 64, 64, engine=request.param, seed=12, ln_noise=0.2, embed_std=0.05)
     yield s
     s.dec.close()
 
@@ -627,12 +642,13 @@ def test_pre_ln_models(name, request):
     assert compared >= 3
 
 
-def test_mbart_full_size_sampled():
+@pytest.mark.parametrize("engine", ["simt", "tensor"])
+def test_mbart_full_size_sampled(engine):
     """The mBART-large-sized preset at its full size (d = 1024, 12 + 12 layers, d_ff = 4096,
     V = 250027, pre-LN, GELU, learned positions): teacher-forced logits of a few rows against
     the oracle, and GS-Jacobi b = 5 / b = 16 equal to greedy with the tokens checked by one
     teacher-forced oracle pass (sampled outputs: the oracle runs the model at full size)."""
-    s = Setup(synth.MBART, 16, 16, seed=0)
+    s = Setup(synth.MBART, 16, 16, engine=engine, seed=0)
     rng = np.random.default_rng(31)
     src = synth.MBART_GS.sentences()[0][:10]
     s.dec.encode(src)
