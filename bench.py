@@ -31,6 +31,7 @@ import synth  # noqa: E402
 
 WORKLOAD = synth.MARIAN_GS
 STOP_RULE = "paper"          # "paper": StopC of Eq. 5; "prefix": accepted-prefix rule
+ENGINE = "auto"              # pd_gemm_engine: auto (SIMT at batch 1, tensor cores batched)
 METRIC = "translated tokens/s at batch 1, GS-Jacobi vs greedy AR; HBM GB/s % of peak"
 FALLBACK_HBM_GBS = 6800.0
 
@@ -245,7 +246,7 @@ def run_gpu(args):
     max_src = max(len(s) for s in sents)
     max_tgt = max(WORKLOAD.max_len(len(s)) for s in sents)
     stream = torch.cuda.Stream()
-    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt), weights.blob,
+    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, engine=ENGINE), weights.blob,
                       stream=stream.cuda_stream)
 
     offs = np.cumsum([0] + [len(s) for s in sents])
@@ -372,7 +373,7 @@ def run_gpu(args):
             "data": "synthetic: seeded N(0,0.02) weights, uniform random source ids",
             "config": {"workload": WORKLOAD.name if n_s == WORKLOAD.n_sentences else
                        f"{WORKLOAD.name} (first {n_s} sentences only)", "sentences_per_step": n_s,
-                       "stop_rule": STOP_RULE,
+                       "stop_rule": STOP_RULE, "engine": ENGINE,
                        "timing": "CUDA events on the library stream; L2 flushed (256 MB write) "
                                  "between steps; replicas across GPUs"},
             "greedy": {"value": greedy_tps, "unit": "tokens/s",
@@ -428,8 +429,8 @@ def run_gpu_batch(args):
     max_src = max(len(s) for s in sents)
     max_tgt = max(WORKLOAD.max_len(len(s)) for s in sents)
     stream = torch.cuda.Stream()
-    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, max_batch=S), weights.blob,
-                      stream=stream.cuda_stream)
+    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, max_batch=S, engine=ENGINE),
+                      weights.blob, stream=stream.cuda_stream)
     offs_all = np.cumsum([0] + [len(s) for s in sents])
     d_src = torch.tensor(np.concatenate(sents), dtype=torch.int32, device="cuda")
     d_y = torch.zeros((len(groups), S, max_tgt), dtype=torch.int32, device="cuda")
@@ -503,7 +504,7 @@ def run_gpu_batch(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic: seeded N(0,0.02) weights, uniform random source ids",
             "config": {"workload": f"{WORKLOAD.name}, batches of {S} sentences",
-                       "sentences_per_step": len(sents), "batch": S, "stop_rule": STOP_RULE,
+                       "sentences_per_step": len(sents), "batch": S, "stop_rule": STOP_RULE, "engine": ENGINE,
                        "timing": "CUDA events on the library stream around encode + decode of "
                                  "all batches; L2 flushed (256 MB write) between steps"},
             "greedy": {"value": greedy_tps, "unit": "tokens/s",
@@ -545,13 +546,16 @@ def main():
                     help="when a block's passes end: paper = StopC of Eq. 5 (the block unchanged, "
                          "or one pass per position); prefix = also once the unchanged leading "
                          "tokens make the whole block exact")
+    ap.add_argument("--engine", default="auto", choices=["auto", "simt", "tensor"],
+                    help="matrix-product engine of the bf16 context (pd_gemm_engine)")
     ap.add_argument("--batch", type=int, default=1,
                     help="sentences decoded together (batched serving); 1 = the batch-1 benchmark")
     ap.add_argument("--sentences", type=int, default=0,
                     help="use only the first N sentences of the workload (profiling runs)")
     args = ap.parse_args()
-    global WORKLOAD, STOP_RULE
+    global WORKLOAD, STOP_RULE, ENGINE
     STOP_RULE = args.stop_rule
+    ENGINE = args.engine
     if args.workload == "marian-knob":
         WORKLOAD = synth.MARIAN_KNOB
     elif args.workload == "mbart":
