@@ -141,9 +141,20 @@ BF16_KNOB = synth.small_spec("post-silu-bf16-knob", d_model=512, n_heads=8, d_ff
 
 # bf16 models run with either matrix-product engine (pd_gemm_engine): the "_tc" fixtures use
 # the tensor cores (tcgen05), the others the SIMT path, each checked against the oracle.
-@pytest.fixture(scope="module", params=["simt", "tensor"])
-def bf16_knob(request):
-    s = Setup(BF16_KNOB, 64, 128, engine=request.param, seed=12, ln_noise=1.0, embed_std=0.012)
+def _bf16_knob(engine):
+    return Setup(BF16_KNOB, 64, 128, engine=engine, seed=12, ln_noise=1.0, embed_std=0.012)
+
+
+@pytest.fixture(scope="module")
+def bf16_knob():
+    s = _bf16_knob("simt")
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
+def bf16_knob_tc():
+    s = _bf16_knob("tensor")
     yield s
     s.dec.close()
 
@@ -298,7 +309,7 @@ def test_marian_logits_bf16(name, request):
         assert rel_row_err(got, ref).max() < 2e-2
 
 
-@pytest.mark.parametrize("name", ["tiny", "bf16_knob", "marian", "marian_tc"])
+@pytest.mark.parametrize("name", ["tiny", "bf16_knob", "bf16_knob_tc", "marian", "marian_tc"])
 def test_logits_batch_invariant(name, request):
     """Batch invariance, the property behind every method's bit identity with greedy: the
     logits of row t (inputs y_0..y_t) are the same bits whether the pass carries t + 1 rows or
@@ -403,11 +414,12 @@ def test_tiny_eos_paths(tiny_eos):
     assert seen_eos >= 2
 
 
-def test_bf16_traces_against_oracle(bf16_knob):
+@pytest.mark.parametrize("name", ["bf16_knob", "bf16_knob_tc"])
+def test_bf16_traces_against_oracle(name, request):
     """bf16 weights: pass counts, per-pass traces and DDGviz probabilities of every method equal
     the oracle's step-by-step runs (all of its decisions clear the bf16 margin), and blocks
     really converge early (fewer passes than positions)."""
-    s = bf16_knob
+    s = request.getfixturevalue(name)
     compared, early = 0, 0
     for src in synth.sentences(22, 3, 6, 12, s.spec.vocab):
         max_len = 2 * len(src)
@@ -423,7 +435,8 @@ def test_bf16_traces_against_oracle(bf16_knob):
     assert early == 3
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_vary", "bf16_knob", "marian", "marian_tc"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_vary", "bf16_knob", "bf16_knob_tc", "marian",
+                                  "marian_tc"])
 def test_trace_probs_against_own_logits_and_oracle(name, request):
     """The DDGviz probability of each greedy pass (softmax probability of the argmax, Section
     3.5) is computed on the device by an online sum of exponentials merged across CTA partials.
@@ -611,14 +624,21 @@ def pre_f32():
     s.dec.close()
 
 
-@pytest.fixture(scope="module", params=["simt", "tensor"])
-def pre_bf16(request):
-    s = Setup(PRE_BF16, 64, 64, engine=request.param, seed=12, ln_noise=0.2, embed_std=0.05)
+@pytest.fixture(scope="module")
+def pre_bf16():
+    s = Setup(PRE_BF16, 64, 64, engine="simt", seed=12, ln_noise=0.2, embed_std=0.05)
     yield s
     s.dec.close()
 
 
-@pytest.mark.parametrize("name", ["pre_f32", "pre_bf16"])
+@pytest.fixture(scope="module")
+def pre_bf16_tc():
+    s = Setup(PRE_BF16, 64, 64, engine="tensor", seed=12, ln_noise=0.2, embed_std=0.05)
+    yield s
+    s.dec.close()
+
+
+@pytest.mark.parametrize("name", ["pre_f32", "pre_bf16", "pre_bf16_tc"])
 def test_pre_ln_models(name, request):
     """Pre-LN blocks with embedding and final LayerNorms, exact GELU and a learned position
     table: logits against the oracle, every method bit-identical to the GPU's greedy, pass
