@@ -421,9 +421,10 @@ __device__ __forceinline__ bool run_gemm(const KParams<W>& P, const GemmArgs<W>&
   if constexpr (TC) {
     const Dims& D = smem_dims<W>();
     const SmemLayout SL = smem_layout(D, sizeof(W));
-    const bool ok = tc_gemm_phase<W>(g, T, D, gph, P.maps,
-                                     smem + SL.ring, smem + SL.bbuf,
-                                     reinterpret_cast<float*>(smem + SL.epi), P.B.red, P.B.cnt);
+    const bool ok = tc_gemm_phase<W>(g, T, D, gph, P.maps, smem + SL.ring, smem + SL.bbuf,
+                                     reinterpret_cast<float*>(smem + SL.epi),
+                                     reinterpret_cast<Partial*>(smem + SL.scratch), P.B.red,
+                                     P.B.cnt);
     if (!ok && threadIdx.x == 0) {
       atomicExch(P.B.bar + 1, 1u);
       atomicCAS(&P.B.st->status, 0, (int)PD_ETIMEOUT);

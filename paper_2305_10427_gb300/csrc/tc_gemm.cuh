@@ -445,10 +445,12 @@ __device__ __forceinline__ void put4_b(unsigned char* bb, int r, int kk, int rti
 
 // Stage rows m0..m0+mt of the GEMM input, K elements k0..k0+KS, into the B layout (rows mt..
 // rtiles*16 zero).  LayerNorm / embedding rows are computed whole (the statistics need the
-// full row); `store` writes the full normalised fp32 rows to g.x_store.
+// full row); `store` writes the full normalised fp32 rows to g.x_store.  lnv: shared memory for
+// the phase's LayerNorm vectors (4 K elements of W).
 template <typename W>
-__device__ void stage_b(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims& D, int m0,
-                        int mt, int k0, int KS, int rtiles, bool store, unsigned char* bb) {
+__device__ __noinline__ void stage_b(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims& D, int m0,
+                        int mt, int k0, int KS, int rtiles, bool store, unsigned char* bb,
+                        W* lnv) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int K = g.K;
@@ -495,45 +497,73 @@ __device__ void stage_b(const GemmArgs<W>& g, const EmbedTabs<W>& T, const Dims&
     }
     return;
   }
-  for (int r = warp; r < mt; r += kWarps) {
-    const int m = m0 + r;
-    const int nI = K / 128;
-    float4 v[kMaxRowRegs];
-    if (g.emb_tok != nullptr) {
-      int t = g.emb_tok[m];
-      t = t < 0 ? 0 : (t >= D.V ? D.V - 1 : t);
-      const int p = g.emb_pos[m];
-      const W* er = T.E + (size_t)t * K;
+  // the LayerNorm vectors of this phase (identical for every row) into shared memory once:
+  // lnv = [ln_a gamma | ln_a beta | ln_b gamma | ln_b beta], K elements each, in W
+  const W *ga_g = g.ln_a_g, *ga_b = g.ln_a_b, *gb_g = g.ln_b_g, *gb_b = g.ln_b_b;
+  if (lnv != nullptr) {
+    const W* src[4] = {g.ln_a_g, g.ln_a_b, g.ln_b_g, g.ln_b_b};
+    const int per = K * (int)sizeof(W) / 16;              // 16-byte chunks per vector
+    for (int f = threadIdx.x; f < 4 * per; f += kThreads) {
+      const int v = f / per, c = f - v * per;
+      if (src[v] != nullptr)
+        *reinterpret_cast<uint4*>(reinterpret_cast<char*>(lnv + (size_t)v * K) + c * 16) =
+            ldg_nc_v4(reinterpret_cast<const char*>(src[v]) + c * 16);
+    }
+    __syncthreads();
+    if (ga_g != nullptr) { ga_g = lnv; ga_b = lnv + K; }
+    if (gb_g != nullptr) { gb_g = lnv + 2 * K; gb_b = lnv + 3 * K; }
+  }
+  // each warp takes two rows at a time (both rows' loads issued before either is normalised)
+  const int nI = K / 128;
+  for (int r0 = warp; r0 < mt; r0 += 2 * kWarps) {
+    float4 v[2][kMaxRowRegs];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int r = r0 + h * kWarps;
+      if (r >= mt) break;
+      const int m = m0 + r;
+      if (g.emb_tok != nullptr) {
+        int t = g.emb_tok[m];
+        t = t < 0 ? 0 : (t >= D.V ? D.V - 1 : t);
+        const int p = g.emb_pos[m];
+        const W* er = T.E + (size_t)t * K;
+#pragma unroll
+        for (int i = 0; i < kMaxRowRegs; ++i) {
+          if (i < nI) {
+            const int k = lane * 4 + 128 * i;
+            const float4 e = get4(er + k);
+            float4 ps;
+            if (T.P != nullptr) ps = get4(T.P + (size_t)(p < D.max_pos ? p : D.max_pos - 1) * K + k);
+            else ps = *reinterpret_cast<const float4*>(T.ptab + (size_t)p * K + k);
+            v[h][i] = make_float4(e.x * D.emb_scale + ps.x, e.y * D.emb_scale + ps.y,
+                                  e.z * D.emb_scale + ps.z, e.w * D.emb_scale + ps.w);
+          }
+        }
+      } else {
+        const float* src = g.x_src + (size_t)m * K;
+#pragma unroll
+        for (int i = 0; i < kMaxRowRegs; ++i)
+          if (i < nI) v[h][i] = *reinterpret_cast<const float4*>(src + lane * 4 + 128 * i);
+      }
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int r = r0 + h * kWarps;
+      if (r >= mt) break;
+      const int m = m0 + r;
+      if (ga_g != nullptr) ln_regs(v[h], nI, K, ga_g, ga_b, D.eps);
+      if (store && g.x_store != nullptr) {
+#pragma unroll
+        for (int i = 0; i < kMaxRowRegs; ++i)
+          if (i < nI)
+            *reinterpret_cast<float4*>(g.x_store + (size_t)m * K + lane * 4 + 128 * i) = v[h][i];
+      }
+      if (gb_g != nullptr) ln_regs(v[h], nI, K, gb_g, gb_b, D.eps);
 #pragma unroll
       for (int i = 0; i < kMaxRowRegs; ++i) {
-        if (i < nI) {
-          const int k = lane * 4 + 128 * i;
-          const float4 e = get4(er + k);
-          float4 ps;
-          if (T.P != nullptr) ps = get4(T.P + (size_t)(p < D.max_pos ? p : D.max_pos - 1) * K + k);
-          else ps = *reinterpret_cast<const float4*>(T.ptab + (size_t)p * K + k);
-          v[i] = make_float4(e.x * D.emb_scale + ps.x, e.y * D.emb_scale + ps.y,
-                             e.z * D.emb_scale + ps.z, e.w * D.emb_scale + ps.w);
-        }
+        const int k = lane * 4 + 128 * i;
+        if (i < nI && k >= k0 && k < k0 + KS) put4_b(bb, r, k - k0, rtiles, v[h][i]);
       }
-    } else {
-      const float* src = g.x_src + (size_t)m * K;
-#pragma unroll
-      for (int i = 0; i < kMaxRowRegs; ++i)
-        if (i < nI) v[i] = *reinterpret_cast<const float4*>(src + lane * 4 + 128 * i);
-    }
-    if (g.ln_a_g != nullptr) ln_regs(v, nI, K, g.ln_a_g, g.ln_a_b, D.eps);
-    if (store && g.x_store != nullptr) {
-#pragma unroll
-      for (int i = 0; i < kMaxRowRegs; ++i)
-        if (i < nI)
-          *reinterpret_cast<float4*>(g.x_store + (size_t)m * K + lane * 4 + 128 * i) = v[i];
-    }
-    if (g.ln_b_g != nullptr) ln_regs(v, nI, K, g.ln_b_g, g.ln_b_b, D.eps);
-#pragma unroll
-    for (int i = 0; i < kMaxRowRegs; ++i) {
-      const int k = lane * 4 + 128 * i;
-      if (i < nI && k >= k0 && k < k0 + KS) put4_b(bb, r, k - k0, rtiles, v[i]);
     }
   }
 }
@@ -575,7 +605,19 @@ __device__ __forceinline__ void epi_store(const GemmArgs<W>& g, const Dims& D, i
   }
 }
 
-constexpr int kArgRows = (kMaxChunk + kWarps - 1) / kWarps;   // chunk rows per warp (argmax)
+// The accumulated values of lane quadrant q (this warp's, q = warp % 4) for the 16-row tile rt:
+// the naccs accumulators summed in a fixed order (v[r] = row 16 rt + r).
+__device__ __forceinline__ void tc_load_acc(uint32_t tmem, int q, int rt, int naccs,
+                                            float (&v)[16]) {
+  const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(rt * kRowTile);
+  tmem_ld16(ta, v);
+  for (int c = 1; c < naccs; ++c) {
+    float w[16];
+    tmem_ld16(ta + (uint32_t)(c * kMaxChunk), w);
+#pragma unroll
+    for (int r = 0; r < 16; ++r) v[r] += w[r];
+  }
+}
 
 // Thread 0: the MMAs of one item over rtiles 16-row tiles.  K-block kb accumulates into
 // accumulator kb % kAccs (tensor-memory columns (kb % kAccs) * kMaxChunk + 16 rt ..), so that
@@ -632,7 +674,7 @@ template <typename W>
 __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTabs<W>& T,
                                            const Dims& D, int gph, const CUtensorMap* maps,
                                            unsigned char* ring, unsigned char* bb, float* epi,
-                                           float* red, unsigned* cnt) {
+                                           Partial* rowp, float* red, unsigned* cnt) {
   TcState& s = smem_tc<W>();
   const PInfo in = s.info[gph];
   const int nj = in.nj, S = in.S, kbs = in.kbs, KS = kbs * kKBlock, N = in.N;
@@ -654,9 +696,9 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
   for (int ch = 0; ch < nch; ++ch) {
     const int m0 = ch * RC, mt = M - m0 < RC ? M - m0 : RC;
     const int rtiles = (mt + kRowTile - 1) / kRowTile;
-    Partial ap[kArgRows];
-#pragma unroll
-    for (int k = 0; k < kArgRows; ++k) ap[k] = Partial{-INFINITY, 0x7fffffff, 0.f, 0};
+    if (argmax)           // the CTA's running argmax partial of each row of the chunk
+      for (int cr = threadIdx.x; cr < mt; cr += kThreads)
+        rowp[cr] = Partial{-INFINITY, 0x7fffffff, 0.f, 0};
     for (int j = 0; j < nj; ++j) {
       const int i = in.first + j * (int)gridDim.x;
       const int tile = S == 1 ? i : i / S, sp = S == 1 ? 0 : i - tile * S;
@@ -665,115 +707,121 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
       const int key = ch * S + sp;
       if (key != staged_key) {
         __syncthreads();                           // the previous MMAs are done (acc wait)
-        stage_b<W>(ga, T, D, m0, mt, sp * KS, KS, rtiles, storer && sp == 0, bb);
+        stage_b<W>(ga, T, D, m0, mt, sp * KS, KS, rtiles, storer && sp == 0, bb,
+                   reinterpret_cast<W*>(epi));
         fence_proxy_async_smem();
         __syncthreads();
         staged_key = key;
       }
-      // per-thread epilogue operand that does not depend on this phase's products
+      // epilogue operands that do not depend on this phase's products: the bias of this
+      // thread's feature (f for the shared-memory path, nfq for the warp-parallel one)
       const int f = threadIdx.x % kTileN;
       const int nf = n0 + f;
+      const int q = warp & 3, nfq = n0 + 32 * q + lane;
       const float bias = (ga.bias != nullptr && nf < N) ? to_f(ga.bias[nf]) : 0.f;
+      const float bq = (ga.bias != nullptr && nfq < N) ? to_f(ga.bias[nfq]) : 0.f;
       if (threadIdx.x == 0) {
         (void)tc_issue_item<W>(D, maps, ring, bb, kbs, rtiles);
         mma_commit(&s.acc);
         (void)mbar_wait(&s.acc, s.acc_n & 1, &s.err);
+        if (!s.err) tc_produce<W>(D, maps, ring, false);   // slots released: stream on
       }
       __syncthreads();
       if (s.err) return false;
       tc_fence_after();
-      for (int rt = 0; rt < rtiles; ++rt) {
-        const int rows = mt - rt * kRowTile < kRowTile ? mt - rt * kRowTile : kRowTile;
-        if (warp < 4) {
-          // the accumulators summed in a fixed order
-          const uint32_t ta = s.tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(rt * kRowTile);
-          float v[16], w[16];
-          tmem_ld16(ta, v);
-          for (int c = 1; c < naccs; ++c) {
-            tmem_ld16(ta + (uint32_t)(c * kMaxChunk), w);
-#pragma unroll
-            for (int r = 0; r < 16; ++r) v[r] += w[r];
-          }
-#pragma unroll
-          for (int r = 0; r < 16; ++r) epi[r * kEpiLd + warp * 32 + lane] = v[r];
-        }
-        __syncthreads();
-        bool mine = true;
+      if (!argmax) {
+        // straight from tensor memory: warp w owns lane quadrant q = w % 4 (features n0 + 32 q
+        // + lane) of the 16-row tiles w / 4, w / 4 + 3, ...; the accumulators are summed in a
+        // fixed order; one thread per feature, so every row's stores are coalesced
+        const size_t rs = (size_t)D.rows;
         if (S > 1) {
-          // split K: publish this slice's partial; the last of the S CTAs to arrive sums the
-          // slices in ascending order and runs the epilogue
-          const size_t rs = (size_t)D.rows;
-          for (int e = threadIdx.x; e < rows * kTileN; e += kThreads) {
-            const int r = e / kTileN, ff = e % kTileN, n = n0 + ff;
-            if (n < N)
-              red[((size_t)sp * rs + m0 + rt * kRowTile + r) * N + n] = epi[r * kEpiLd + ff];
+          // split K: publish this slice's partial; the last of the S CTAs to arrive for this
+          // tile and chunk sums the slices in ascending order and runs the epilogue
+          for (int rt = warp >> 2; rt < rtiles; rt += kWarps / 4) {
+            float v[16];
+            tc_load_acc(s.tmem, q, rt, naccs, v);
+            const int rows = mt - rt * kRowTile < kRowTile ? mt - rt * kRowTile : kRowTile;
+            if (nfq < N)
+              for (int r = 0; r < rows; ++r)
+                red[((size_t)sp * rs + m0 + rt * kRowTile + r) * N + nfq] = v[r];
           }
           __threadfence();
           __syncthreads();
           if (threadIdx.x == 0) {
             unsigned* c = cnt + (size_t)(tile * ((D.rows + kRowTile - 1) / kRowTile) +
-                                         (m0 + rt * kRowTile) / kRowTile) % kCounterSlots;
+                                         m0 / kRowTile) % kCounterSlots;
             const unsigned old = atomicAdd(c, 1u);
             s.last = old == (unsigned)(S - 1);
             if (s.last) atomicExch(c, 0u);
           }
           __syncthreads();
-          mine = s.last != 0;
-          if (mine) {
+          if (s.last) {
             __threadfence();
-            for (int e = threadIdx.x; e < rows * kTileN; e += kThreads) {
-              const int r = e / kTileN, ff = e % kTileN, n = n0 + ff;
-              float acc = 0.f;
-              if (n < N)
-                for (int q = 0; q < S; ++q)
-                  acc += __ldcg(red + ((size_t)q * rs + m0 + rt * kRowTile + r) * N + n);
-              epi[r * kEpiLd + ff] = acc;
+            for (int rt = warp >> 2; rt < rtiles; rt += kWarps / 4) {
+              const int rows = mt - rt * kRowTile < kRowTile ? mt - rt * kRowTile : kRowTile;
+              if (nfq < N)
+                for (int r = 0; r < rows; ++r) {
+                  const int m = m0 + rt * kRowTile + r;
+                  float acc = 0.f;
+                  for (int qq = 0; qq < S; ++qq) acc += __ldcg(red + ((size_t)qq * rs + m) * N + nfq);
+                  const float resid = ga.epi == EPI_RESID ? ga.resid[(size_t)m * ga.ld + nfq] : 0.f;
+                  epi_store<W>(ga, D, m, nfq, acc, bq, resid);
+                }
             }
-            __syncthreads();
           }
-        }
-        if (mine) {
-          if (argmax) {
-            // warp w keeps the running partials of chunk rows w, w + 12, ...; lane l takes
-            // features l, l + 32, l + 64, l + 96 of the tile
+        } else {
+          for (int rt = warp >> 2; rt < rtiles; rt += kWarps / 4) {
+            float v[16];
+            tc_load_acc(s.tmem, q, rt, naccs, v);
+            const int rows = mt - rt * kRowTile < kRowTile ? mt - rt * kRowTile : kRowTile;
+            if (nfq < N)
 #pragma unroll
-            for (int k = 0; k < kArgRows; ++k) {
-              const int cr = warp + k * kWarps;
-              const int r = cr - rt * kRowTile;
-              if (r >= 0 && r < rows) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                  const int ff = lane + 32 * q, n = n0 + ff;
-                  if (n < N)
-                    argmax_push(epi[r * kEpiLd + ff], n, ap[k].mx, ap[k].idx, ap[k].sum,
-                                ap[k].nan);
+              for (int r = 0; r < 16; ++r) {
+                if (r < rows) {
+                  const int m = m0 + rt * kRowTile + r;
+                  const float resid = ga.epi == EPI_RESID ? ga.resid[(size_t)m * ga.ld + nfq] : 0.f;
+                  epi_store<W>(ga, D, m, nfq, v[r], bq, resid);
                 }
               }
-            }
-          } else if (nf < N) {
-            // thread -> feature f = tid % 128 (one bias value), rows tid / 128 + 3 u
-            for (int r = threadIdx.x / kTileN; r < rows; r += kThreads / kTileN) {
-              const int m = m0 + rt * kRowTile + r;
-              const float resid = ga.epi == EPI_RESID ? ga.resid[(size_t)m * ga.ld + nf] : 0.f;
-              epi_store<W>(ga, D, m, nf, epi[r * kEpiLd + f], bias, resid);
-            }
           }
         }
-        __syncthreads();
+      } else {
+        // LM head argmax: the tile goes through shared memory, one 16-row tile at a time
+        for (int rt = 0; rt < rtiles; ++rt) {
+          const int rows = mt - rt * kRowTile < kRowTile ? mt - rt * kRowTile : kRowTile;
+          if (warp < 4) {
+            float v[16];
+            tc_load_acc(s.tmem, warp, rt, naccs, v);
+#pragma unroll
+            for (int r = 0; r < 16; ++r) epi[r * kEpiLd + warp * 32 + lane] = v[r];
+          }
+          __syncthreads();
+          // row r of the tile -> warp r % 12; lane l takes features l, l + 32, l + 64, l + 96,
+          // the lanes' partials meet in a fixed butterfly, and lane 0 merges the item's partial
+          // into the row's running one (items in ascending order)
+          for (int r = warp; r < rows; r += kWarps) {
+            Partial a{-INFINITY, 0x7fffffff, 0.f, 0};
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+              const int ff = lane + 32 * qq, n = n0 + ff;
+              if (n < N) argmax_push(epi[r * kEpiLd + ff], n, a.mx, a.idx, a.sum, a.nan);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) partial_merge(a, shfl_partial(a, o));
+            if (lane == 0) partial_merge(rowp[rt * kRowTile + r], a);
+          }
+          __syncthreads();
+        }
       }
+      (void)bias;
       tc_fence_before();
       __syncthreads();
       if (threadIdx.x == 0) s.acc_n += 1;
     }
     if (argmax) {
-#pragma unroll
-      for (int k = 0; k < kArgRows; ++k) {
-        const int cr = warp + k * kWarps;
-        Partial a = ap[k];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) partial_merge(a, shfl_partial(a, o));
-        if (lane == 0 && cr < mt) ga.part[(size_t)blockIdx.x * ga.part_ld + m0 + cr] = a;
-      }
+      __syncthreads();
+      for (int cr = threadIdx.x; cr < mt; cr += kThreads)
+        ga.part[(size_t)blockIdx.x * ga.part_ld + m0 + cr] = rowp[cr];
     }
   }
   __syncthreads();
