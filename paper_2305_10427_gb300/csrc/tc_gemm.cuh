@@ -623,7 +623,8 @@ __device__ __forceinline__ void tc_load_acc(uint32_t tmem, int q, int rt, int na
 // accumulator kb % kAccs (tensor-memory columns (kb % kAccs) * kMaxChunk + 16 rt ..), so that
 // kAccs dependent chains of MMAs run side by side; within a chain the K-blocks and the K = 16
 // steps are in ascending order.  Every K-block's slot is released by a commit once its MMAs
-// are done.  Returns false if the weight stream or a wait failed.
+// are done (the stream is topped up after the item, while the CTA waits at barriers, and on
+// demand when a block has not been issued yet).  Returns false if a wait failed.
 template <typename W>
 __device__ __forceinline__ bool tc_issue_item(const Dims& D, const CUtensorMap* maps,
                                               unsigned char* ring, unsigned char* bb, int kbs,
@@ -660,7 +661,6 @@ __device__ __forceinline__ bool tc_issue_item(const Dims& D, const CUtensorMap* 
                (kb >= kAccs || k16 > 0) ? 1u : 0u);
     mma_commit(&s.empty[slot]);
     cseq += 1;
-    tc_produce<W>(D, maps, ring, false);
   }
   s.c_seq = cseq;
   return ok;
