@@ -74,6 +74,9 @@ typedef struct {
   int max_batch;     /* capacity: sentences one pd_encode_batch / pd_decode_batch carries,
                         0 or 1..64 (0 = 1); each needs its own key/value caches */
   int gemm_engine;   /* pd_gemm_engine: how the bf16 matrix products run (fp32: always SIMT) */
+  int kv_pages;      /* capacity of each decoder layer's self-attention key/value pool, in
+                        pages of 16 positions (0 = max_batch * ceil(max_tgt_len / 16)); a
+                        decode needs sum over its sentences of ceil(max_len / 16) pages */
 } pd_config;
 
 /* How a bf16 context runs the matrix products of its encoder and decoder passes.  Every pass of

@@ -46,7 +46,7 @@ class _Config(ctypes.Structure):
                                             "eos_id", "bos_id")] + \
               [("ln_eps", ctypes.c_float), ("max_src_len", ctypes.c_int),
                ("max_tgt_len", ctypes.c_int), ("max_batch", ctypes.c_int),
-               ("gemm_engine", ctypes.c_int)]
+               ("gemm_engine", ctypes.c_int), ("kv_pages", ctypes.c_int)]
 
 
 class _DecodeParams(ctypes.Structure):
@@ -138,15 +138,16 @@ class Config:
     max_tgt_len: int = 256
     max_batch: int = 0
     gemm_engine: int = 0
+    kv_pages: int = 0
 
     @classmethod
     def from_spec(cls, spec, max_src_len: int, max_tgt_len: int, pad_id=1, eos_id=0, bos_id=2,
-                  max_batch: int = 0, engine: str = "auto"):
+                  max_batch: int = 0, engine: str = "auto", kv_pages: int = 0):
         """Build from any object carrying the model fields (d_model, n_heads, ...)."""
         return cls(spec.d_model, spec.n_heads, spec.d_ff, spec.n_enc_layers, spec.n_dec_layers,
                    spec.vocab, spec.activation, bool(spec.pre_ln), bool(spec.learned_pos),
                    spec.max_pos, spec.dtype, pad_id, eos_id, bos_id, spec.ln_eps, max_src_len,
-                   max_tgt_len, max_batch, ENGINES[engine])
+                   max_tgt_len, max_batch, ENGINES[engine], kv_pages)
 
     def _c(self) -> _Config:
         c = _Config()

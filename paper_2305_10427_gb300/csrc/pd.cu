@@ -64,19 +64,26 @@ struct SmemLayout {
 
 // The commit region: per pass row r (at most D.rows) its new token (-1 for a NaN row) and
 // probability, and the row's description (input token, position, self-attention cache slot,
-// first slot of its sentence, keys it attends, first cross key row and cross key count); per
-// sentence its decoding state, its first row in the pass and y_0..y_m.
+// its sentence, keys it attends, first cross key row and cross key count); per sentence its
+// decoding state, its first row in the pass, y_0..y_m and its page table (the pool page of
+// each 16 positions of its self-attention keys and values).
 struct CommitMem {
   int *ntok, *rtok, *rpos, *rslot, *rsb, *rkn, *rxb, *rxn;
   float* nprob;
   DecState* st;
   int* r0;
   int* y;                   // [max_batch][max_tgt + 1]
+  int* pt;                  // [max_batch][pt_ld]
   int* misc;                // [0] rows of the current pass
 };
 __host__ __device__ inline size_t commit_bytes(const Dims& D) {
   return (size_t)D.rows * 9 * 4 + (size_t)D.max_batch * (sizeof(DecState) + 4) +
-         (size_t)D.max_batch * (D.max_tgt + 1) * 4 + 64;
+         (size_t)D.max_batch * (D.max_tgt + 1) * 4 + (size_t)D.max_batch * D.pt_ld * 4 + 64;
+}
+
+// Cache slot of position pos of the sentence whose page table is pt.
+__device__ __forceinline__ int page_slot(const int* pt, int pos) {
+  return pt[pos >> kPageShift] * kPageRows + (pos & (kPageRows - 1));
 }
 __device__ __forceinline__ CommitMem commit_mem(const Dims& D, unsigned char* base) {
   CommitMem c;
@@ -93,6 +100,7 @@ __device__ __forceinline__ CommitMem commit_mem(const Dims& D, unsigned char* ba
   c.st = reinterpret_cast<DecState*>(p); p += D.max_batch * (int)(sizeof(DecState) / 4);
   c.r0 = p; p += D.max_batch;
   c.y = p; p += D.max_batch * (D.max_tgt + 1);
+  c.pt = p; p += D.max_batch * D.pt_ld;
   c.misc = p;
   return c;
 }
@@ -319,8 +327,8 @@ __device__ void gemm_args(const KParams<W>& P, int ph, int M, const int* rtok, c
         else { g.ln_a_g = mw.dec[l - 1].ln3g; g.ln_a_b = mw.dec[l - 1].ln3b; g.x_store = B.xa; }
       }
       g.w = L.wqkv; g.bias = L.bqkv; g.epi = EPI_QKV; g.out = B.q; g.ld = D.d;
-      g.kdst = B.kself + (size_t)l * D.max_batch * D.max_tgt * D.d;
-      g.vdst = B.vself + (size_t)l * D.max_batch * D.max_tgt * D.d;
+      g.kdst = B.kself + (size_t)l * D.kv_pages * kPageRows * D.d;
+      g.vdst = B.vself + (size_t)l * D.kv_pages * kPageRows * D.d;
       g.slot = rslot;
       break;
     case PH_O:                          // self-attention output + residual
@@ -472,7 +480,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
   // TMA loads would queue behind bulk L2 prefetches in the same copy engine)
   if constexpr (!TC) prefetch_pass_start(P);
   __syncthreads();
-  const size_t self_ld = (size_t)D.max_batch * D.max_tgt * D.d;
+  const size_t self_ld = (size_t)D.kv_pages * kPageRows * D.d;
   const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
   for (int ph = 0; ph < nph; ++ph) {
     const bool attn = is_attn_phase(ph, nph);
@@ -480,7 +488,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
       const int l = ph >> 3;
       if ((ph & 7) == PH_SELF)
         attn_phase<W, W>(D, B.q, B.kself + l * self_ld, B.vself + l * self_ld, B.att, M,
-                         cm.rsb, cm.rkn, 0, scratch);
+                         cm.rsb, cm.rkn, 0, scratch, cm.pt);
       else
         attn_phase<W, W>(D, B.q, B.kcross + l * cross_ld, B.vcross + l * cross_ld, B.att, M,
                          cm.rxb, cm.rxn, 0, scratch);
@@ -529,8 +537,8 @@ __device__ void build_rows(const KParams<W>& P, const CommitMem& cm) {
       const int r = cm.r0[s] + j, pos = st.i - 1 + j;
       cm.rtok[r] = ys[pos];
       cm.rpos[r] = pos;
-      cm.rsb[r] = s * D.max_tgt;
-      cm.rslot[r] = s * D.max_tgt + pos;
+      cm.rsb[r] = s;
+      cm.rslot[r] = page_slot(cm.pt + s * D.pt_ld, pos);
       cm.rkn[r] = pos + 1;                  // block-causal: keys 0..pos of its own sentence
       cm.rxb[r] = s * D.max_src;
       cm.rxn[r] = st.n_src;
@@ -657,7 +665,7 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   }
   __syncthreads();
   for (int r = tid; r < M; r += blockDim.x)        // y_{i:i+blk} <- new, every sentence
-    cm.y[(size_t)(cm.rsb[r] / D.max_tgt) * (D.max_tgt + 1) + cm.rpos[r] + 1] = cm.ntok[r];
+    cm.y[(size_t)cm.rsb[r] * (D.max_tgt + 1) + cm.rpos[r] + 1] = cm.ntok[r];
   __syncthreads();
   for (int s = tid; s < S; s += blockDim.x) {      // the first EOS among y_1..y_m ends y
     DecState& st = cm.st[s];
@@ -717,10 +725,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   const CommitMem cm = commit_mem(D, smem + SL.commit);
   if constexpr (TC) tc_setup<W>(D, TC_DECODE, SL.ring_slots, P.maps);
 
+  for (int e = threadIdx.x; e < D.max_batch * D.pt_ld; e += blockDim.x) cm.pt[e] = B.page_tab[e];
+  __syncthreads();
+
   if (P.debug_len > 0) {                  // teacher-forced rows 0..len-1 of the slot-0 sentence
     for (int m = threadIdx.x; m < P.debug_len; m += blockDim.x) {
       cm.rtok[m] = B.dbg_tok[m];
-      cm.rpos[m] = m; cm.rslot[m] = m; cm.rsb[m] = 0; cm.rkn[m] = m + 1;
+      cm.rpos[m] = m; cm.rslot[m] = page_slot(cm.pt, m); cm.rsb[m] = 0; cm.rkn[m] = m + 1;
       cm.rxb[m] = 0; cm.rxn[m] = P.n_src_s[0];
     }
     __syncthreads();
@@ -900,6 +911,7 @@ struct pd_ctx {
   int64_t launches = 0;
   float* static_logits = nullptr;              // device address of the fixed logits array
   std::vector<CUtensorMap> dec_maps, enc_maps; // bf16: per GEMM phase of each kernel
+  std::vector<int32_t> page_host;              // the sentences' page tables of the last decode
   std::string err;
 };
 
@@ -941,6 +953,9 @@ bool valid_config(const pd_config* c, std::string* why) {
   if (!(c->ln_eps >= 0.f)) return bad("ln_eps");
   if (c->max_batch < 0 || c->max_batch > pd::kMaxBatch) return bad("max_batch must be in [0, 64]");
   if (c->gemm_engine < PD_ENGINE_AUTO || c->gemm_engine > PD_ENGINE_TENSOR) return bad("gemm_engine");
+  if (c->kv_pages != 0 &&
+      (c->kv_pages < (c->max_tgt_len + pd::kPageRows - 1) / pd::kPageRows || c->kv_pages > (1 << 20)))
+    return bad("kv_pages must be 0 or hold one sentence of max_tgt_len (<= 2^20 pages)");
   if (c->dtype == PD_DTYPE_BF16 && c->vocab < pd::kTileN)
     return bad("bf16 models need vocab >= 128 (one tensor-core tile)");
   return true;
@@ -1144,8 +1159,10 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
   PD_TRY(dalloc(c, &B.att, R * d));
   PD_TRY(dalloc(c, &B.ffh, R * (size_t)D.f));
   const size_t nb = (size_t)D.max_batch;
-  PD_TRY(dalloc(c, &B.kself, (size_t)D.Ld * nb * D.max_tgt * d));
-  PD_TRY(dalloc(c, &B.vself, (size_t)D.Ld * nb * D.max_tgt * d));
+  PD_TRY(dalloc(c, &B.kself, (size_t)D.Ld * D.kv_pages * pd::kPageRows * d));
+  PD_TRY(dalloc(c, &B.vself, (size_t)D.Ld * D.kv_pages * pd::kPageRows * d));
+  PD_TRY(dalloc(c, &B.page_tab, nb * D.pt_ld));
+  c->page_host.assign(nb * D.pt_ld, 0);
   PD_TRY(dalloc(c, &B.kcross, (size_t)D.Ld * nb * D.max_src * d));
   PD_TRY(dalloc(c, &B.vcross, (size_t)D.Ld * nb * D.max_src * d));
   PD_TRY(dalloc(c, &B.part, (size_t)c->grid * R));
@@ -1228,6 +1245,8 @@ pd_status encode_impl(pd_ctx* c, const int32_t* d_src, int n, int slot, bool res
   return PD_OK;
 }
 
+pd_status assign_pages(pd_ctx* c, int n_sent, const int32_t* len, int len_all);
+
 // max_len: per-sentence values (host), or nullptr for p->max_len everywhere
 template <typename W>
 pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int n_sent, const int32_t* max_len,
@@ -1245,6 +1264,7 @@ pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int n_sent, const in
   P.out_y = d_y;
   P.out_ld = y_ld;
   P.out_info = d_info;
+  PD_TRY(assign_pages(c, n_sent, max_len, p->max_len));
   return launch<W>(c, false, P);
 }
 
@@ -1252,6 +1272,7 @@ pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int n_sent, const in
 // it (PD_ETIMEOUT) is the only status the caller can read back afterwards (debug_status).
 template <typename W>
 pd_status debug_impl(pd_ctx* c, int len, float* d_logits) {
+  PD_TRY(assign_pages(c, 1, nullptr, len));
   pd::KParams<W> P = base_params<W>(c);
   P.debug_len = len;
   P.logits = d_logits;
@@ -1267,6 +1288,37 @@ pd_status debug_status(pd_ctx* c) {
   PD_CUDA(c, cudaMemcpy(&st, &dst->status, sizeof(int), cudaMemcpyDeviceToHost));
   if (st != 0) return fail(c, (pd_status)st, "the teacher-forced pass stopped early (a device "
                                              "wait gave up); no logits were returned");
+  return PD_OK;
+}
+
+// Page tables of a decode: sentence s needs ceil(len_s / 16) pages of the self-attention
+// key/value pool (positions 0..len_s - 1 are written); pages are handed out round robin over
+// the sentences (page j of every sentence, then page j + 1, ...), so a sentence's pages are not
+// contiguous in the pool.  The tables go to the device on the context stream.
+pd_status assign_pages(pd_ctx* c, int n_sent, const int32_t* len, int len_all) {
+  const Dims& D = c->D;
+  long need = 0;
+  int most = 0;
+  for (int s = 0; s < n_sent; ++s) {
+    const int l = len ? len[s] : len_all;
+    const int np = (l + pd::kPageRows - 1) / pd::kPageRows;
+    need += np;
+    most = std::max(most, np);
+  }
+  if (need > D.kv_pages)
+    return fail(c, PD_EINVAL, "the key/value page pool (kv_pages = " + std::to_string(D.kv_pages) +
+                                  ") is smaller than the " + std::to_string(need) +
+                                  " pages these sentences need");
+  int next = 0;
+  for (int j = 0; j < most; ++j)
+    for (int s = 0; s < n_sent; ++s) {
+      const int l = len ? len[s] : len_all;
+      if (j < (l + pd::kPageRows - 1) / pd::kPageRows) c->page_host[(size_t)s * D.pt_ld + j] = next++;
+    }
+  int* dtab = c->cfg.dtype == PD_DTYPE_BF16 ? c->bb.page_tab : c->bf.page_tab;
+  PD_CUDA(c, cudaMemcpyAsync(dtab, c->page_host.data(),
+                             (size_t)n_sent * D.pt_ld * sizeof(int32_t), cudaMemcpyHostToDevice,
+                             c->stream));
   return PD_OK;
 }
 
@@ -1339,6 +1391,8 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   D.max_src = cfg->max_src_len; D.max_tgt = cfg->max_tgt_len;
   D.max_keys = D.max_src > D.max_tgt ? D.max_src : D.max_tgt;
   D.max_batch = cfg->max_batch > 1 ? cfg->max_batch : 1;
+  D.pt_ld = (D.max_tgt + pd::kPageRows - 1) / pd::kPageRows;
+  D.kv_pages = cfg->kv_pages > 0 ? cfg->kv_pages : D.max_batch * D.pt_ld;
   const long batch_rows = std::min<long>((long)D.max_batch * D.max_tgt, pd::kMaxPassRows);
   D.rows = (int)std::max<long>(D.max_keys, batch_rows);
   D.tc = cfg->dtype == PD_DTYPE_BF16 &&

@@ -27,6 +27,8 @@ constexpr int kNCol = 4;            // output columns per warp iteration (kNCol 
 constexpr int kMaxLayers = 16;
 constexpr int kMaxBatch = 64;        // sentences of one batched decode
 constexpr int kMaxPassRows = 512;    // rows of one batched decoder pass
+constexpr int kPageShift = 4;        // self-attention key/value cache pages of 16 positions
+constexpr int kPageRows = 1 << kPageShift;
 constexpr unsigned long long kWaitNs = 10000000000ull;  // bounded device waits: 10 s
 
 enum Epi : int {
@@ -68,6 +70,8 @@ struct Dims {
   int max_batch;   // sentences one decode carries (cache slots per layer)
   int rows;        // activation rows: max(max_keys, min(max_batch * max_tgt, kMaxPassRows))
   int tc;          // bf16: GEMM phases on the tensor cores (else the SIMT path)
+  int kv_pages;    // pages of kPageRows cache rows in each decoder layer's self K/V pool
+  int pt_ld;       // page-table entries per sentence: ceil(max_tgt / kPageRows)
 };
 
 // Per-CTA partial of the LM-head argmax for one row.
@@ -98,7 +102,8 @@ struct Bufs {
   float *q, *k, *v;            // [rows][d]
   W* att;                      // [rows][d] attention output, rounded to W (the O input type)
   W* ffh;                      // [rows][f] FFN hidden, rounded to W (FFN2's input type)
-  W *kself, *vself;            // [Ld][max_batch * max_tgt][d]: sentence s at slots s * max_tgt..
+  W *kself, *vself;            // [Ld][kv_pages * kPageRows][d]: pages of 16 positions, found
+                               // through each sentence's page table
   W *kcross, *vcross;          // [Ld][max_batch * max_src][d]: sentence s at rows s * max_src..
   Partial* part;               // [grid][rows]
   DecState* st;
@@ -109,6 +114,8 @@ struct Bufs {
   int* src;                    // [max_src]
   int* dbg_tok;                // [max_tgt]
   float* pos_tab;              // sinusoidal positions [rows][d] (built once at create)
+  int* page_tab;               // [max_batch][pt_ld] pool page of each sentence's 16-position
+                               // page (written by the host before a decode)
   float* red;                  // bf16: split-K partial sums [S][rows][N]
   unsigned* cnt;               // bf16: split-K arrival counters (zero between uses)
 };
@@ -769,13 +776,21 @@ __device__ __forceinline__ void add_pv32(const float* v, float p, float (&acc)[3
 // One warp per (row m, head): lane l owns keys l, l+32, ...  Scores, softmax and the
 // p-weighted value sums are accumulated per lane in ascending key order, then combined by
 // fixed butterflies, so a row's result depends only on its own query and keys.
-// Row m attends the rkeys[m] keys starting at key row rbase[m] of kc / vc (its sentence's
-// cache: causal rows pass their position + 1); without the arrays every row attends the first
-// n_keys keys.
+// Row m attends rkeys[m] keys of kc / vc (causal rows pass their position + 1); without the
+// arrays every row attends the first n_keys keys.  Key j of row m is at key row rbase[m] + j
+// (contiguous caches), or, given a page table ptab ([sentence][pt_ld], the paged self-attention
+// cache), rbase[m] is the row's sentence s and key j sits in pool page ptab[s][j / 16] at
+// row j % 16.
+template <typename KV>
+__device__ __forceinline__ size_t key_row(const int* ptab, int pt_ld, int base, int j) {
+  return ptab != nullptr
+             ? (size_t)ptab[base * pt_ld + (j >> kPageShift)] * kPageRows + (j & (kPageRows - 1))
+             : (size_t)base + j;
+}
 template <typename KV, typename O>
 __device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV* kc, const KV* vc,
                            O* out, int M, const int* rbase, const int* rkeys, int n_keys,
-                           float* scratch) {
+                           float* scratch, const int* ptab = nullptr) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int gw = warp * gridDim.x + blockIdx.x;     // items dealt to CTAs round robin
@@ -787,12 +802,12 @@ __device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV*
   for (int it = gw; it < M * D.H; it += tw) {
     const int m = it / D.H, h = it - m * D.H;
     const int T = rkeys != nullptr ? rkeys[m] : n_keys;
-    const size_t kb = rbase != nullptr ? (size_t)rbase[m] * D.d : 0;
+    const int base = rbase != nullptr ? rbase[m] : 0;
     for (int e = lane; e < dh; e += 32) qs[e] = q[(size_t)m * D.d + h * dh + e] * scale;
     __syncwarp();
     float lmax = -INFINITY;
     for (int j = lane; j < T; j += 32) {
-      const float s = key_dot<KV>(kc + kb + (size_t)j * D.d + h * dh, qs, dh);
+      const float s = key_dot<KV>(kc + key_row<KV>(ptab, D.pt_ld, base, j) * D.d + h * dh, qs, dh);
       ps[j] = s;
       lmax = fmaxf(lmax, s);
     }
@@ -810,7 +825,7 @@ __device__ __noinline__ void attn_phase(const Dims& D, const float* q, const KV*
       for (int e = 0; e < 32; ++e) acc[e] = 0.f;
       for (int j = lane; j < T; j += 32) {
         const float p = ps[j];
-        add_pv32(vc + kb + (size_t)j * D.d + h * dh + c0, p, acc);
+        add_pv32(vc + key_row<KV>(ptab, D.pt_ld, base, j) * D.d + h * dh + c0, p, acc);
       }
       const float tot = reduce_scatter32(acc);
       out[(size_t)m * D.d + h * dh + c0 + lane] = from_f<O>(tot / sum);

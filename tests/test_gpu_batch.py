@@ -125,3 +125,32 @@ def test_batch_errors():
     assert e.value.status == -1
     assert len(dec.decode_batch("jacobi", [60] * 8)) == 8       # 480 rows
     dec.close()
+
+
+@pytest.mark.parametrize("engine", ["simt", "tensor"])
+def test_paged_cache_pool(engine):
+    """The self-attention keys and values live in a pool of 16-position pages handed out per
+    decode (sentence s's pages interleaved with the others', never contiguous in a batch).  A
+    pool sized for the batch's actual lengths (here 12 pages instead of the 4 x 8 that max_tgt_len
+    would need) decodes every sentence exactly as a context with the default pool decodes it
+    alone, and a request that needs more pages than the pool holds is rejected before any
+    launch."""
+    spec = synth.TINY if engine == "simt" else MODELS["marian"][0]
+    w = synth.make_weights(spec, seed=0)
+    big = pkg.Decoder(pkg.Config.from_spec(spec, 64, 128, engine=engine), w.blob)
+    small = pkg.Decoder(pkg.Config.from_spec(spec, 64, 128, max_batch=4, engine=engine,
+                                             kv_pages=12), w.blob)
+    sents = synth.sentences(65, 4, 8, 20, spec.vocab)
+    max_len = [min(48, 2 * len(s)) for s in sents]          # <= 3 pages each, 12 in all
+    small.encode_batch(sents)
+    for m, b in (("gs_jacobi", 5), ("jacobi", 0), ("greedy", 1)):
+        got = small.decode_batch(m, max_len, b=b)
+        for k, s in enumerate(sents):
+            big.encode(s)
+            ref = big.decode(m, max_len[k], b=b)
+            assert (got[k].tokens, got[k].n_iters) == (ref.tokens, ref.n_iters), (m, k)
+    with pytest.raises(pkg.PdError) as e:
+        small.decode_batch("greedy", [64, 64, 64, 64])         # 16 pages > 12
+    assert e.value.status == -1 and "page pool" in str(e.value)
+    small.close()
+    big.close()
