@@ -131,7 +131,20 @@ pd_status pd_encode_device(pd_ctx* ctx, const int32_t* d_src, int n_src);
  *    already equal to the solution), so the whole block is, and the confirming pass that
  *    Eq. 5 needs is skipped.  The paper leaves other stopping conditions to future work
  *    (Section 5, Conclusions); this is one, with the same result and at most as many passes. */
-typedef enum { PD_STOP_UNCHANGED = 0, PD_STOP_PREFIX = 1 } pd_stop_rule;
+typedef enum { PD_STOP_UNCHANGED = 0, PD_STOP_PREFIX = 1, PD_STOP_SUFFIX = 2 } pd_stop_rule;
+
+/* PD_STOP_SUFFIX: the accepted-prefix rule, with each further pass of a block re-running only
+ * the block positions after its exact prefix (the first c + 1 new tokens of the last pass):
+ * the same tokens, passes and trace as PD_STOP_PREFIX (the rows it skips would reproduce their
+ * tokens bit for bit), fewer rows per pass.  The paper names other stopping conditions and
+ * cheaper iterations as future work (Section 5). */
+
+/* The drafts a new block of Jacobi / GS-Jacobi / Hybrid GS-Jacobi starts from (InitT,
+ * Section 3.3).  PD_INIT_PAD: every draft is PAD, as in the paper.  PD_INIT_LAST: every draft
+ * is the last token already decided, y_{i-1} (one of the other initialisations the paper
+ * leaves to future work, Section 5).  Proposition 1 holds for any initialisation: the tokens are
+ * the greedy ones either way; the pass counts differ. */
+typedef enum { PD_INIT_PAD = 0, PD_INIT_LAST = 1 } pd_init_rule;
 
 typedef struct {
   int method;       /* pd_method */
@@ -142,14 +155,16 @@ typedef struct {
   int stop_at_eos;  /* greedy / jacobi / gs_jacobi: end the returned y at the first EOS */
   int max_passes;   /* 0 = no limit; else stop with PD_ENOTCONV after this many passes */
   int stop_rule;    /* pd_stop_rule (0 = Eq. 5) */
+  int init;         /* pd_init_rule (0 = PAD, the paper's InitT) */
 } pd_decode_params;
 
 /* One decoder pass of the trace (DDGviz-style, Section 3.5): pass number (1-based), block
  * start position i (1-based), block length, number of leading block positions whose new
- * token equals the previous draft, StopC (Eq. 5) flag (under either stop rule), index of the
- * first EOS in the new block tokens (-1 if none). */
+ * token equals the previous draft, StopC (Eq. 5) flag (under any stop rule), index of the
+ * first EOS in the new block tokens (-1 if none), rows the pass computed (block_len, or fewer
+ * under PD_STOP_SUFFIX). */
 typedef struct {
-  int32_t step, block_start, block_len, n_converged, stop, eos_idx;
+  int32_t step, block_start, block_len, n_converged, stop, eos_idx, n_rows;
 } pd_trace_step;
 
 /* Decode the sentence last given to pd_encode.  Outputs (host): y[0..*n_y) = y_1..y_m

@@ -18,6 +18,15 @@ Readings of the paper that this file fixes (each one listed in the design notes)
   EOS or max_len.
 * Jacobi and GS-Jacobi solve the system for a known m (Section 4.1 "we assume to know
   beforehand the length m"); with ``stop_at_eos`` the returned tokens end at the first EOS.
+
+Options the paper leaves to future work (Section 5, other initialisations and stopping
+conditions), with the same solution by Proposition 1:
+
+* ``stop_rule="prefix"``: a block also ends once the first c + 1 new tokens of a pass (c the
+  unchanged leading count) cover it; ``stop_rule="suffix"``: the same, and every further pass
+  of a block computes only the positions after that exact prefix.
+* ``init_rule="last"``: a new block's drafts are the last decided token y_{i-1} repeated
+  instead of PAD (greedy steps and Hybrid's greedy tail have no drafts to initialise).
 """
 from __future__ import annotations
 
@@ -54,6 +63,7 @@ class TraceRow:
     tokens: List[int]
     probs: Optional[List[float]] = None
     min_margin: float = float("inf")
+    n_rows: int = 0              # rows the pass computed (fewer than block_len: suffix rule)
 
 
 @dataclasses.dataclass
@@ -98,7 +108,8 @@ def greedy(step: Step, max_len: int, stop_at_eos: bool = True, bos: int = synth.
         mm = float(out.margin[i - 1]) if out.margin is not None else float("inf")
         pr = [float(out.prob[i - 1])] if out.prob is not None else None
         same = int(tok == pad)                    # the one-position "block" vs its PAD draft
-        trace.append(TraceRow(i, i, 1, same, bool(same), 0 if tok == eos else -1, [tok], pr, mm))
+        trace.append(TraceRow(i, i, 1, same, bool(same), 0 if tok == eos else -1, [tok], pr, mm,
+                              n_rows=1))
         if stop_at_eos and tok == eos:
             break
     return Result(y[1:], len(trace), trace)
@@ -107,32 +118,38 @@ def greedy(step: Step, max_len: int, stop_at_eos: bool = True, bos: int = synth.
 def _block_passes(step: Step, y: List[int], i: int, blk: int, n_pass: int, trace: List[TraceRow],
                   eos: int, stop_rule: str):
     """Repeat one decoder pass over the block y_i..y_{i+blk-1} until the stopping condition
-    (Eq. 5: the block did not change) or the pass cap; returns the updated pass counter."""
+    (Eq. 5: the block did not change) or the pass cap; returns the updated pass counter.
+    Under the suffix rule a pass takes new tokens only for the block positions after the
+    exact prefix a (the first c + 1 tokens of the pass before); positions below a keep theirs."""
+    a = 0
     for k in range(1, blk + 1):
         o = list(y[i:i + blk])                          # copy(y_{i:i+b})
         out = step(y[:i + blk - 1])                     # inputs y_0..y_{i+b-2}
-        new = [int(t) for t in out.pred[i - 1:i - 1 + blk]]
+        new = o[:a] + [int(t) for t in out.pred[i - 1 + a:i - 1 + blk]]
         y[i:i + blk] = new                              # y_{i:i+b} <- argmax p(. | y_{1:i+b}, x)
         n_pass += 1
         c = _leading_equal(o, new)
         stop = c == blk                                 # StopC(o, y_{i:i+b})
-        mm = float(np.min(out.margin[i - 1:i - 1 + blk])) if out.margin is not None \
+        mm = float(np.min(out.margin[i - 1 + a:i - 1 + blk])) if out.margin is not None \
             else float("inf")
         pr = [float(p) for p in out.prob[i - 1:i - 1 + blk]] if out.prob is not None else None
-        trace.append(TraceRow(n_pass, i, blk, c, stop, _first(new, eos), new, pr, mm))
+        trace.append(TraceRow(n_pass, i, blk, c, stop, _first(new, eos), new, pr, mm,
+                              n_rows=blk - a))
         if stop:
             break
-        if stop_rule == "prefix" and c + 1 >= blk:
+        if stop_rule in ("prefix", "suffix") and c + 1 >= blk:
             break
+        if stop_rule == "suffix":
+            a = c + 1
     return n_pass
 
 
 def gs_jacobi(step: Step, m: int, b: int, init: Optional[Sequence[int]] = None,
-              stop_at_eos: bool = True, stop_rule: str = "paper",
+              stop_at_eos: bool = True, stop_rule: str = "paper", init_rule: str = "pad",
               bos: int = synth.BOS_ID, pad: int = synth.PAD_ID, eos: int = synth.EOS_ID) -> Result:
     """Algorithm 2 (Parallel GS-Jacobi): Jacobi passes inside blocks of b positions, blocks
     solved one after the other (Gauss-Seidel across blocks).  InitT = all PAD unless ``init``
-    gives another draft of length m."""
+    gives another draft of length m, or ``init_rule="last"`` re-initialises each block."""
     if b < 1:
         raise ValueError("b must be >= 1")
     y = [bos] + (list(init) if init is not None else [pad] * m)
@@ -143,6 +160,8 @@ def gs_jacobi(step: Step, m: int, b: int, init: Optional[Sequence[int]] = None,
     i = 1
     while i <= m:
         blk = min(b, m - i + 1)
+        if init_rule == "last":
+            y[i:i + blk] = [y[i - 1]] * blk
         n_pass = _block_passes(step, y, i, blk, n_pass, trace, eos, stop_rule)
         i += blk
     out = y[1:]
@@ -157,7 +176,7 @@ def jacobi(step: Step, m: int, init: Optional[Sequence[int]] = None, stop_at_eos
 
 def hybrid_gs_jacobi(step: Step, max_len: int, b: int, h: Optional[int] = None,
                      init: Optional[Sequence[int]] = None, stop_rule: str = "paper",
-                     bos: int = synth.BOS_ID, pad: int = synth.PAD_ID,
+                     init_rule: str = "pad", bos: int = synth.BOS_ID, pad: int = synth.PAD_ID,
                      eos: int = synth.EOS_ID) -> Result:
     """Algorithm 3 (Hybrid GS-Jacobi): GS-Jacobi blocks up to length h (default max_len); a
     finished block that contains EOS ends decoding with the prefix through that EOS;
@@ -169,6 +188,8 @@ def hybrid_gs_jacobi(step: Step, max_len: int, b: int, h: Optional[int] = None,
     i = 1
     while i <= h:
         blk = min(b, h - i + 1)
+        if init_rule == "last":
+            y[i:i + blk] = [y[i - 1]] * blk
         n_pass = _block_passes(step, y, i, blk, n_pass, trace, eos, stop_rule)
         e = _first(y[i:i + blk], eos)
         if e >= 0:
@@ -184,7 +205,7 @@ def hybrid_gs_jacobi(step: Step, max_len: int, b: int, h: Optional[int] = None,
         pr = [float(out.prob[i - 1])] if out.prob is not None else None
         same = int(tok == pad)
         trace.append(TraceRow(n_pass, i, 1, same, bool(same), 0 if tok == eos else -1, [tok], pr,
-                              mm))
+                              mm, n_rows=1))
         i += 1
         if tok == eos:
             break
@@ -192,16 +213,19 @@ def hybrid_gs_jacobi(step: Step, max_len: int, b: int, h: Optional[int] = None,
 
 
 def decode(step: Step, method: str, max_len: int, b: int = 1, h: Optional[int] = None,
-           stop_at_eos: bool = True, init=None, stop_rule: str = "paper") -> Result:
+           stop_at_eos: bool = True, init=None, stop_rule: str = "paper",
+           init_rule: str = "pad") -> Result:
     if method == "greedy":
         return greedy(step, max_len, stop_at_eos)
     if method == "jacobi":
-        return jacobi(step, max_len, init=init, stop_at_eos=stop_at_eos, stop_rule=stop_rule)
+        return jacobi(step, max_len, init=init, stop_at_eos=stop_at_eos, stop_rule=stop_rule,
+                      init_rule=init_rule)
     if method == "gs_jacobi":
         return gs_jacobi(step, max_len, b, init=init, stop_at_eos=stop_at_eos,
-                         stop_rule=stop_rule)
+                         stop_rule=stop_rule, init_rule=init_rule)
     if method == "hybrid_gs_jacobi":
-        return hybrid_gs_jacobi(step, max_len, b, h=h, init=init, stop_rule=stop_rule)
+        return hybrid_gs_jacobi(step, max_len, b, h=h, init=init, stop_rule=stop_rule,
+                                init_rule=init_rule)
     raise ValueError(method)
 
 

@@ -22,7 +22,9 @@ STATUS_NAMES = {0: "PD_OK", -1: "PD_EINVAL", -2: "PD_ENOMEM", -3: "PD_ECUDA", -4
                 -5: "PD_ENAN", -6: "PD_ESTATE", -7: "PD_ETIMEOUT"}
 
 METHODS = {"greedy": 0, "jacobi": 1, "gs_jacobi": 2, "hybrid_gs_jacobi": 3}
-STOP_RULES = {"paper": 0, "prefix": 1}      # pd_stop_rule: Eq. 5 StopC, accepted prefix
+STOP_RULES = {"paper": 0, "prefix": 1, "suffix": 2}   # pd_stop_rule: Eq. 5 StopC, accepted
+#                                                     prefix, accepted prefix with suffix re-runs
+INITS = {"pad": 0, "last": 1}                         # pd_init_rule
 ENGINES = {"auto": 0, "simt": 1, "tensor": 2}   # pd_gemm_engine
 
 # Every symbol include/pd.h declares.
@@ -51,12 +53,12 @@ class _Config(ctypes.Structure):
 
 class _DecodeParams(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in ("method", "b", "max_len", "h", "stop_at_eos",
-                                            "max_passes", "stop_rule")]
+                                            "max_passes", "stop_rule", "init")]
 
 
 class _TraceStep(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in ("step", "block_start", "block_len", "n_converged",
-                                              "stop", "eos_idx")]
+                                              "stop", "eos_idx", "n_rows")]
 
 
 _lib = None
@@ -226,12 +228,12 @@ class Decoder:
 
     def decode_batch(self, method: str, max_len, b: int = 1, h: int = 0,
                      stop_at_eos: bool = True, max_passes: int = 0,
-                     stop_rule: str = "paper") -> List["DecodeResult"]:
+                     stop_rule: str = "paper", init: str = "pad") -> List["DecodeResult"]:
         """Decode the sentences of the last encode_batch together; max_len: one value per
         sentence."""
         ml = np.ascontiguousarray(max_len, dtype=np.int32)
         n = ml.size
-        p = self.params(method, int(ml.max()), b, h, stop_at_eos, max_passes, stop_rule)
+        p = self.params(method, int(ml.max()), b, h, stop_at_eos, max_passes, stop_rule, init)
         y_ld = int(ml.max())
         y = np.zeros((n, y_ld), dtype=np.int32)
         n_y = np.zeros(n, dtype=np.int32)
@@ -250,14 +252,14 @@ class Decoder:
 
     @staticmethod
     def params(method: str, max_len: int, b: int = 1, h: int = 0, stop_at_eos: bool = True,
-               max_passes: int = 0, stop_rule: str = "paper") -> _DecodeParams:
+               max_passes: int = 0, stop_rule: str = "paper", init: str = "pad") -> _DecodeParams:
         return _DecodeParams(METHODS[method], int(b), int(max_len), int(h), int(stop_at_eos),
-                             int(max_passes), STOP_RULES[stop_rule])
+                             int(max_passes), STOP_RULES[stop_rule], INITS[init])
 
     def decode(self, method: str, max_len: int, b: int = 1, h: int = 0,
                stop_at_eos: bool = True, max_passes: int = 0,
-               trace: bool = False, stop_rule: str = "paper") -> DecodeResult:
-        p = self.params(method, max_len, b, h, stop_at_eos, max_passes, stop_rule)
+               trace: bool = False, stop_rule: str = "paper", init: str = "pad") -> DecodeResult:
+        p = self.params(method, max_len, b, h, stop_at_eos, max_passes, stop_rule, init)
         y = np.zeros(max_len, dtype=np.int32)
         n_y, n_it, n_tr = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
         if trace:

@@ -514,7 +514,8 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
 
 // Rows of the next pass: every sentence that is not done contributes its block rows, inputs
 // y_{i-1} then the draft at positions i-1..i+blk-2 (the shift-left of Algorithm 2's appendix
-// note), sentences in order.  All threads of the CTA; misc[0] = the row count.
+// note; under the suffix rule only the rows after the block's exact prefix), sentences in
+// order.  All threads of the CTA; misc[0] = the row count.
 template <typename W>
 __device__ void build_rows(const KParams<W>& P, const CommitMem& cm) {
   const Dims& D = smem_dims<W>();
@@ -523,18 +524,29 @@ __device__ void build_rows(const KParams<W>& P, const CommitMem& cm) {
     int r = 0;
     for (int s = 0; s < S; ++s) {
       cm.r0[s] = r;
-      if (!cm.st[s].done) r += cm.st[s].blk;
+      if (!cm.st[s].done) r += cm.st[s].blk - cm.st[s].a;
     }
     cm.misc[0] = r;
   }
-  __syncthreads();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  // a fresh block's drafts under the last-token rule: y_{i-1} repeated (else they stay PAD)
+  for (int s = warp; s < S; s += kWarps) {
+    const DecState& st = cm.st[s];
+    if (st.done || st.k != 0 || st.init_rule != PD_INIT_LAST || st.method == PD_GREEDY ||
+        st.ar_tail)
+      continue;
+    int* ys = cm.y + (size_t)s * (D.max_tgt + 1);
+    const int last = ys[st.i - 1];
+    for (int j = lane; j < st.blk; j += 32) ys[st.i + j] = last;
+  }
+  __syncthreads();
   for (int s = warp; s < S; s += kWarps) {
     const DecState& st = cm.st[s];
     if (st.done) continue;
     const int* ys = cm.y + (size_t)s * (D.max_tgt + 1);
-    for (int j = lane; j < st.blk; j += 32) {
-      const int r = cm.r0[s] + j, pos = st.i - 1 + j;
+    // rows predict block offsets a..blk-1 (a > 0 only under the suffix rule)
+    for (int j = lane; j < st.blk - st.a; j += 32) {
+      const int r = cm.r0[s] + j, pos = st.i - 1 + st.a + j;
       cm.rtok[r] = ys[pos];
       cm.rpos[r] = pos;
       cm.rsb[r] = s;
@@ -592,17 +604,19 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
   for (int s = tid; s < S; s += blockDim.x) {
     DecState st = cm.st[s];                        // decisions on a register copy
     if (st.done) continue;
-    const int r0 = cm.r0[s], blk = st.blk, i = st.i;
-    const int* nt = cm.ntok + r0;
+    const int r0 = cm.r0[s], blk = st.blk, i = st.i, a = st.a;
+    const int* nt = cm.ntok + r0 - a;              // the pass's rows are block offsets a..blk-1
     const int* ys = cm.y + (size_t)s * (D.max_tgt + 1);
+    // the block's new tokens: offsets below a were exact before this pass and stay as they are
+    auto newtok = [&](int off) { return off < a ? ys[i + off] : nt[off]; };
     bool nan = false;
-    for (int r = 0; r < blk; ++r) nan = nan || nt[r] < 0;
-    int c = 0;                                     // leading positions equal to the old draft
+    for (int r = a; r < blk; ++r) nan = nan || nt[r] < 0;
+    int c = a;                                     // leading positions equal to the old draft
     while (c < blk && nt[c] == ys[i + c]) ++c;
     const int stop = c == blk;
     int eos_idx = -1;
     for (int r = 0; r < blk; ++r)
-      if (nt[r] == D.eos) { eos_idx = r; break; }
+      if (newtok(r) == D.eos) { eos_idx = r; break; }
     st.k = st.k + 1;
     const int n_it = st.n_iters + 1;
     st.n_iters = n_it;
@@ -611,11 +625,13 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
       if (S == 1 && blockIdx.x == 0) {
         pd_trace_step row;
         row.step = n_it; row.block_start = i; row.block_len = blk; row.n_converged = c;
-        row.stop = stop; row.eos_idx = eos_idx;
+        row.stop = stop; row.eos_idx = eos_idx; row.n_rows = blk - a;
         B.trace[t] = row;
         for (int r = 0; r < blk; ++r) {
-          B.trace_tok[(size_t)t * D.max_tgt + r] = nt[r];
-          B.trace_prob[(size_t)t * D.max_tgt + r] = cm.nprob[r0 + r];
+          B.trace_tok[(size_t)t * D.max_tgt + r] = newtok(r);
+          // a row not re-run keeps the probability of the pass that made it exact
+          B.trace_prob[(size_t)t * D.max_tgt + r] =
+              r < a ? B.trace_prob[(size_t)(t - 1) * D.max_tgt + r] : cm.nprob[r0 + r - a];
         }
       }
       st.n_trace = t + 1;
@@ -623,13 +639,15 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
     if (nan) {
       st.status = PD_ENAN; st.n_y = i - 1; st.done = 1;
     } else {
-      // the block is solved: StopC, the pass cap, or (accepted-prefix rule) the first c + 1
-      // new tokens exact with c + 1 >= blk
-      if (stop || st.k >= blk || (st.stop_rule == PD_STOP_PREFIX && c + 1 >= blk)) {
+      // the block is solved: StopC, the pass cap, or (accepted-prefix and suffix rules) the
+      // first c + 1 new tokens exact with c + 1 >= blk
+      const bool prefix = st.stop_rule == PD_STOP_PREFIX || st.stop_rule == PD_STOP_SUFFIX;
+      if (stop || st.k >= blk || (prefix && c + 1 >= blk)) {
+        st.a = 0;
         const bool one_pos = st.method == PD_GREEDY || st.ar_tail;
         if (one_pos) {
           const bool eos_ends = st.ar_tail ? true : (st.stop_at_eos != 0);
-          if (eos_ends && nt[0] == D.eos) { st.n_y = i; st.done = 1; }
+          if (eos_ends && newtok(0) == D.eos) { st.n_y = i; st.done = 1; }
         } else if (st.method == PD_HYBRID_GS_JACOBI && eos_idx >= 0) {
           st.n_y = i + eos_idx;                    // through the EOS (Algorithm 3)
           st.done = 1;
@@ -652,6 +670,8 @@ __device__ __noinline__ void commit(const KParams<W>& P, unsigned char* smem) {
             st.k = 0;
           }
         }
+      } else if (st.stop_rule == PD_STOP_SUFFIX) {
+        st.a = c + 1;                              // the next pass re-runs offsets c+1..blk-1
       }
       // the pass budget, and a hard cap no correct schedule reaches (at most m passes for the
       // parallel part plus max_len for a greedy tail): the loop can never run away
@@ -752,7 +772,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     st.i = 1;
     st.blk = st.b_eff < st.m_eff ? st.b_eff : st.m_eff;
     st.k = 0; st.ar_tail = 0; st.n_iters = 0; st.done = 0; st.n_y = 0; st.n_trace = 0;
-    st.status = 0; st.scan = 0;
+    st.status = 0; st.scan = 0; st.a = 0;
     cm.st[s] = st;
   }
   for (int e = threadIdx.x; e < S * (D.max_tgt + 1); e += blockDim.x)
@@ -1259,6 +1279,7 @@ pd_status decode_impl(pd_ctx* c, const pd_decode_params* p, int n_sent, const in
   P.init.stop_at_eos = p->stop_at_eos;
   P.init.max_passes = p->max_passes;
   P.init.stop_rule = p->stop_rule;
+  P.init.init_rule = p->init;
   P.n_sent = n_sent;
   for (int s = 0; s < n_sent; ++s) P.max_len_s[s] = max_len ? max_len[s] : p->max_len;
   P.out_y = d_y;
@@ -1330,8 +1351,10 @@ pd_status check_params(pd_ctx* c, const pd_decode_params* p, int n_sent = 1,
   if ((p->method == PD_GS_JACOBI || p->method == PD_HYBRID_GS_JACOBI) && p->b < 1)
     return fail(c, PD_EINVAL, "b must be >= 1");
   if (p->max_passes < 0) return fail(c, PD_EINVAL, "max_passes must be >= 0");
-  if (p->stop_rule != PD_STOP_UNCHANGED && p->stop_rule != PD_STOP_PREFIX)
+  if (p->stop_rule != PD_STOP_UNCHANGED && p->stop_rule != PD_STOP_PREFIX &&
+      p->stop_rule != PD_STOP_SUFFIX)
     return fail(c, PD_EINVAL, "stop_rule");
+  if (p->init != PD_INIT_PAD && p->init != PD_INIT_LAST) return fail(c, PD_EINVAL, "init");
   if (n_sent < 1 || n_sent > c->D.max_batch) return fail(c, PD_EINVAL, "n_sent must be in [1, max_batch]");
   long rows = 0;                                  // rows of the widest pass
   for (int s = 0; s < n_sent; ++s) {

@@ -93,6 +93,8 @@ struct DecState {
   int n_iters, done, status, n_y, n_trace;
   int n_src;              // source length of the sentence (cross-attention keys)
   int scan;               // the first EOS of y_1..y_m is still to be found
+  int a;                  // suffix rule: block positions i..i+a-1 already exact (not re-run)
+  int init_rule;          // pd_init_rule: drafts of a new block
 };
 
 template <typename W>

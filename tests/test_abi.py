@@ -133,6 +133,12 @@ def test_binding_enums_match_header():
         "PD_GS_JACOBI": B.METHODS["gs_jacobi"],
         "PD_HYBRID_GS_JACOBI": B.METHODS["hybrid_gs_jacobi"]}
     assert _enum_values(text, "pd_stop_rule") == {"PD_STOP_UNCHANGED": B.STOP_RULES["paper"],
-                                                  "PD_STOP_PREFIX": B.STOP_RULES["prefix"]}
+                                                  "PD_STOP_PREFIX": B.STOP_RULES["prefix"],
+                                                  "PD_STOP_SUFFIX": B.STOP_RULES["suffix"]}
+    assert _enum_values(text, "pd_init_rule") == {"PD_INIT_PAD": B.INITS["pad"],
+                                                  "PD_INIT_LAST": B.INITS["last"]}
+    assert _enum_values(text, "pd_gemm_engine") == {"PD_ENGINE_AUTO": B.ENGINES["auto"],
+                                                    "PD_ENGINE_SIMT": B.ENGINES["simt"],
+                                                    "PD_ENGINE_TENSOR": B.ENGINES["tensor"]}
     status = _enum_values(text, "pd_status")
     assert {v: k for k, v in status.items()} == B.STATUS_NAMES

@@ -226,8 +226,8 @@ def assert_same_run(got, ref, name, scales=None, bar=None):
     assert len(got.trace) == len(ref.trace), name
     for t, (a, r) in enumerate(zip(got.trace, ref.trace)):
         assert (a["step"], a["block_start"], a["block_len"], a["n_converged"], bool(a["stop"]),
-                a["eos_idx"]) == (r.step, r.block_start, r.block_len, r.n_converged, r.stop,
-                                  r.eos_idx), (name, t)
+                a["eos_idx"], a["n_rows"]) == (r.step, r.block_start, r.block_len, r.n_converged,
+                                               r.stop, r.eos_idx, r.n_rows), (name, t)
         blk = a["block_len"]
         assert list(got.trace_tokens[t][:blk]) == r.tokens, (name, t)
         if scales is not None and r.probs is not None:
@@ -349,12 +349,49 @@ def test_tiny_all_methods(name, request):
 PREFIX_RUNS = (("jacobi", 0), ("gs_jacobi", 3), ("gs_jacobi", 5), ("hybrid_gs_jacobi", 3))
 
 
-def oracle_run(step, method, max_len, b, eos, rule):
+def oracle_run(step, method, max_len, b, eos, rule, init_rule="pad"):
     if method == "jacobi":
-        return od.jacobi(step, max_len, eos=eos, stop_rule=rule)
+        return od.jacobi(step, max_len, eos=eos, stop_rule=rule, init_rule=init_rule)
     if method == "gs_jacobi":
-        return od.gs_jacobi(step, max_len, b, eos=eos, stop_rule=rule)
-    return od.hybrid_gs_jacobi(step, max_len, b, eos=eos, stop_rule=rule)
+        return od.gs_jacobi(step, max_len, b, eos=eos, stop_rule=rule, init_rule=init_rule)
+    return od.hybrid_gs_jacobi(step, max_len, b, eos=eos, stop_rule=rule, init_rule=init_rule)
+
+
+@pytest.mark.parametrize("name", ["tiny_vary", "tiny_eos", "tiny_fast", "bf16_knob",
+                                  "bf16_knob_tc"])
+def test_suffix_rule_and_last_token_init(name, request):
+    """Options the paper leaves to future work (Section 5): the suffix-only re-run (same
+    passes and trace as the accepted-prefix rule, fewer rows: n_rows in the trace) and the
+    last-token InitT (y_{i-1} repeated as a new block's drafts).  Every run returns the GPU's
+    greedy tokens, and equals the oracle's run of the same rule and initialisation (tokens,
+    passes, trace with rows) wherever the oracle's decisions had margin."""
+    s = request.getfixturevalue(name)
+    srcs = synth.sentences(24, 3, 5, 14, s.spec.vocab)
+    compared = fewer = 0
+    for src in srcs:
+        max_len = 2 * len(src)
+        s.dec.encode(src)
+        g = s.dec.decode("greedy", max_len)
+        step = s.step(src)
+        for m, b in PREFIX_RUNS:
+            runs = {}
+            for rule, init in (("prefix", "pad"), ("suffix", "pad"), ("paper", "last"),
+                               ("suffix", "last")):
+                r = s.dec.decode(m, max_len, b=b, trace=True, stop_rule=rule, init=init)
+                assert r.tokens == g.tokens, (m, b, rule, init)
+                runs[rule, init] = r
+                ref = oracle_run(step, m, max_len, b, s.eos, rule, init)
+                if ref.min_margin > s.margin:
+                    assert_same_run(r, ref, (m, b, rule, init))
+                    compared += 1
+            pre, suf = runs["prefix", "pad"], runs["suffix", "pad"]
+            key = lambda t: [tuple(v for k, v in row.items() if k != "n_rows") for row in t.trace]
+            assert key(suf) == key(pre) and suf.n_iters == pre.n_iters
+            rows_pre = sum(t["n_rows"] for t in pre.trace)
+            rows_suf = sum(t["n_rows"] for t in suf.trace)
+            assert rows_suf <= rows_pre
+            fewer += rows_suf < rows_pre
+    assert compared >= 4 and fewer >= 1
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny_vary", "tiny_eos", "tiny_fast"])
@@ -475,8 +512,15 @@ def test_marian_methods_bit_identical(name, request):
             r = marian.dec.decode(m, max_len, b=b)
             assert r.tokens == g.tokens, (m, b)
             assert r.n_iters <= max_len
+            for rule, init in (("suffix", "pad"), ("paper", "last"), ("suffix", "last")):
+                o = marian.dec.decode(m, max_len, b=b, stop_rule=rule, init=init)
+                assert o.tokens == g.tokens, (m, b, rule, init)
+                assert o.n_iters <= max_len
+        last = marian.dec.decode("gs_jacobi", max_len, b=5, init="last")
         frac = check_tokens_teacher_forced(marian, src, g.tokens)
-        print(f"marian sentence of {len(src)} ids: {frac:.3f} of positions checked")
+        print(f"marian sentence of {len(src)} ids: {frac:.3f} of positions checked; "
+              f"GS-Jacobi b=5 passes from PAD / from the last token: "
+              f"{marian.dec.decode('gs_jacobi', max_len, b=5).n_iters} / {last.n_iters}")
         assert frac >= MARIAN_MIN_COVERED
 
 

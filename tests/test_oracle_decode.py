@@ -264,3 +264,74 @@ def test_planted_missing_cap_breaks_pass_count(monkeypatch):
     monkeypatch.setattr(od, "_block_passes", uncapped)
     r = od.gs_jacobi(chain, 10, 5, stop_at_eos=False)
     assert r.n_iters != 10                      # the closed form (blk per block) catches it
+
+
+# ---- options the paper leaves to future work: suffix re-runs, last-token InitT ---------------
+
+def copy_model(inputs):
+    """y_p = y_{p-1}: every prediction copies its input token (what the random-weight presets
+    do), so the solution is BOS repeated and a draft of y_{i-1} repeated is already exact."""
+    return od.StepOut(np.array(list(inputs)))
+
+
+def _trace_key(r):
+    return [(t.step, t.block_start, t.block_len, t.n_converged, t.stop, t.eos_idx, t.tokens)
+            for t in r.trace]
+
+
+@pytest.mark.parametrize("m,b", [(1, 1), (7, 3), (10, 5), (12, 4), (16, 16)])
+def test_last_token_init_closed_form(m, b):
+    """Copy model: from PAD every block is a dependency chain (blk passes); from y_{i-1}
+    repeated the first pass already returns the draft, StopC holds, one pass per block."""
+    blocks = _blocks(m, b)
+    g = od.greedy(copy_model, m, stop_at_eos=False)
+    assert g.tokens == [BOS] * m
+    for rule in ("paper", "prefix", "suffix"):
+        pad = od.gs_jacobi(copy_model, m, b, stop_rule=rule, stop_at_eos=False)
+        last = od.gs_jacobi(copy_model, m, b, stop_rule=rule, stop_at_eos=False,
+                            init_rule="last")
+        assert pad.tokens == last.tokens == g.tokens
+        assert pad.n_iters == sum(blocks)
+        assert last.n_iters == len(blocks)
+        assert all(t.stop and t.n_converged == t.block_len for t in last.trace)
+    # a chain whose map has no fixed point gains nothing from the last token
+    assert od.gs_jacobi(chain, m, b, stop_at_eos=False, init_rule="last").n_iters == sum(blocks)
+
+
+@pytest.mark.parametrize("m,b", [(7, 3), (10, 5), (12, 4), (16, 16)])
+def test_suffix_rule_equals_prefix_rule_with_fewer_rows(m, b):
+    """The suffix rule re-runs only the positions after a block's exact prefix: the same
+    tokens, passes and trace as the accepted-prefix rule; on a chain a block of k positions
+    computes k + (k-1) + ... + 1 rows instead of k per pass."""
+    for step in (position_only(), chain, skip_chain, copy_model, position_only(eos_at=5)):
+        for init_rule in ("pad", "last"):
+            pre = od.gs_jacobi(step, m, b, stop_rule="prefix", stop_at_eos=False,
+                               init_rule=init_rule)
+            suf = od.gs_jacobi(step, m, b, stop_rule="suffix", stop_at_eos=False,
+                               init_rule=init_rule)
+            assert _trace_key(suf) == _trace_key(pre)
+            assert all(s.n_rows <= p.n_rows == p.block_len for s, p in zip(suf.trace, pre.trace))
+    r = od.gs_jacobi(chain, m, b, stop_rule="suffix", stop_at_eos=False)
+    assert sum(t.n_rows for t in r.trace) == sum(k * (k + 1) // 2 for k in _blocks(m, b))
+    h_pre = od.hybrid_gs_jacobi(position_only(eos_at=6), m, b, stop_rule="prefix")
+    h_suf = od.hybrid_gs_jacobi(position_only(eos_at=6), m, b, stop_rule="suffix")
+    assert _trace_key(h_suf) == _trace_key(h_pre)
+
+
+@pytest.mark.parametrize("toy", TOYS, ids=lambda t: t[0].name)
+def test_proposition_1_new_options(toy):
+    """Any InitT and stop rule reach the greedy solution within m passes (Proposition 1) on the
+    brute-force toy transformers."""
+    m_len = 9
+    for seed in range(2):
+        model, src = _toy(toy, seed)
+        step = od.model_step(model, src)
+        g = od.greedy(step, m_len, stop_at_eos=False)
+        ge = od.greedy(step, m_len)
+        for rule in ("paper", "prefix", "suffix"):
+            for b in (1, 2, 3, m_len):
+                r = od.gs_jacobi(step, m_len, b, stop_at_eos=False, stop_rule=rule,
+                                 init_rule="last")
+                assert r.tokens == g.tokens and r.n_iters <= m_len
+            r = od.hybrid_gs_jacobi(step, m_len, 3, stop_rule=rule, init_rule="last")
+            assert r.tokens == ge.tokens and r.n_iters <= m_len
