@@ -32,6 +32,7 @@ import synth  # noqa: E402
 WORKLOAD = synth.MARIAN_GS
 STOP_RULE = "paper"          # "paper": StopC of Eq. 5; "prefix": accepted-prefix rule
 ENGINE = "auto"              # pd_gemm_engine: auto (SIMT at batch 1, tensor cores batched)
+ARGS_WORKLOAD = "marian"
 METRIC = "translated tokens/s at batch 1, GS-Jacobi vs greedy AR; HBM GB/s % of peak"
 FALLBACK_HBM_GBS = 6800.0
 
@@ -185,6 +186,28 @@ def oracle_tokens_per_s(weights, sentences, budget_s):
     return tokens / dt, tokens, dt, used
 
 
+def oracle_one_thread(budget_s, shortest_first=True):
+    """The oracle timed with one BLAS thread, in a child process (the thread count of a BLAS
+    library is fixed when it loads); returns (tokens/s, tokens, seconds, sentences used)."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    cmd = [sys.executable, os.path.abspath(__file__), "--oracle-worker",
+           "--cpu-budget", str(budget_s), "--workload", ARGS_WORKLOAD]
+    out = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=600)
+    if out.returncode != 0:
+        raise RuntimeError("one-thread oracle run failed: " + out.stderr[-500:])
+    d = json.loads(out.stdout.strip().splitlines()[-1])
+    return d["value"], d["tokens"], d["seconds"], d["used"]
+
+
+def run_oracle_worker(args):
+    sents = WORKLOAD.sentences()
+    order = sorted(range(len(sents)), key=lambda k: len(sents[k]))
+    v, t, d, used = oracle_tokens_per_s(WORKLOAD.weights(), [sents[k] for k in order],
+                                        args.cpu_budget)
+    print(json.dumps({"value": v, "tokens": t, "seconds": d, "used": len(used)}), flush=True)
+    return 0
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -258,6 +281,13 @@ def run_gpu(args):
                   for s in sents]
               for m, b in (("gs_jacobi", WORKLOAD.b), ("greedy", 1), ("jacobi", 1),
                            ("hybrid_gs_jacobi", 3))}
+    # options the paper leaves to future work: suffix-only re-runs, last-token InitT
+    params["gs_jacobi+suffix"] = [pkg.Decoder.params("gs_jacobi", WORKLOAD.max_len(len(s)),
+                                                     b=WORKLOAD.b, stop_rule="suffix")
+                                  for s in sents]
+    params["gs_jacobi+init_last"] = [pkg.Decoder.params("gs_jacobi", WORKLOAD.max_len(len(s)),
+                                                        b=WORKLOAD.b, stop_rule=STOP_RULE,
+                                                        init="last") for s in sents]
 
     def device_step(method, ev=None):
         for k in range(n_s):
@@ -311,7 +341,7 @@ def run_gpu(args):
     # the other methods (one timed step each), for the report
     others = {}
     if args.all_methods:
-        for m in ("jacobi", "hybrid_gs_jacobi"):
+        for m in ("jacobi", "hybrid_gs_jacobi", "gs_jacobi+suffix", "gs_jacobi+init_last"):
             t_tok, t_ms, _, _, t_info = timed(m, 1, 1)
             others[m] = {"value": sum_over_ranks(t_tok) / (max_over_ranks(t_ms) / 1e3),
                          "unit": "tokens/s",
@@ -364,6 +394,10 @@ def run_gpu(args):
         cpu = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"{len(used)} shortest sentences of the 256 ({t} tokens, {d:.1f} s), "
                          f"GS-Jacobi b=5, numpy float64, BLAS threads = all cores"}
+        v1, t1, d1, u1 = oracle_one_thread(args.cpu_budget / 2)
+        cpu["one_thread"] = {"value": v1, "unit": "tokens/s", "cores": 1,
+                             "sample": f"{u1} shortest sentences ({t1} tokens, {d1:.1f} s), "
+                                       f"one BLAS thread"}
 
     if rank == 0:
         line = {
@@ -546,6 +580,7 @@ def main():
                     help="when a block's passes end: paper = StopC of Eq. 5 (the block unchanged, "
                          "or one pass per position); prefix = also once the unchanged leading "
                          "tokens make the whole block exact")
+    ap.add_argument("--oracle-worker", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--engine", default="auto", choices=["auto", "simt", "tensor"],
                     help="matrix-product engine of the bf16 context (pd_gemm_engine)")
     ap.add_argument("--batch", type=int, default=1,
@@ -553,9 +588,10 @@ def main():
     ap.add_argument("--sentences", type=int, default=0,
                     help="use only the first N sentences of the workload (profiling runs)")
     args = ap.parse_args()
-    global WORKLOAD, STOP_RULE, ENGINE
+    global WORKLOAD, STOP_RULE, ENGINE, ARGS_WORKLOAD
     STOP_RULE = args.stop_rule
     ENGINE = args.engine
+    ARGS_WORKLOAD = args.workload
     if args.workload == "marian-knob":
         WORKLOAD = synth.MARIAN_KNOB
     elif args.workload == "mbart":
@@ -563,6 +599,8 @@ def main():
     if args.b and args.b != WORKLOAD.b:
         WORKLOAD = dataclasses.replace(
             WORKLOAD, b=args.b, name=WORKLOAD.name.replace(f"b={WORKLOAD.b}", f"b={args.b}"))
+    if args.oracle_worker:
+        return run_oracle_worker(args)
     if args.impl == "reference":
         return run_reference(args)
     if args.batch > 1:

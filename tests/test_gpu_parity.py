@@ -14,6 +14,8 @@ Checks, per the method's guarantees:
   statuses (bad arguments, decode before encode, pass budget, NaN weights).
 """
 import ctypes
+import os
+import sys
 
 import numpy as np
 import pytest
@@ -22,6 +24,8 @@ import synth
 import paper_2305_10427_gb300 as pkg
 from oracle import decode as od
 from oracle import model as om
+
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
 
 pytestmark = pytest.mark.gpu
 
@@ -728,3 +732,33 @@ def test_mbart_full_size_sampled(engine):
         assert r.n_iters <= 12
     check_tokens_teacher_forced(s, src, g.tokens)
     s.dec.close()
+
+
+def test_ddgviz_dump_of_a_gpu_decode(tiny_vary, tmp_path):
+    """The DDGviz-style JSONL dump of a GPU decode (Section 3.5): the records round-trip, carry
+    the trace field by field, and their settle passes equal those of the oracle's run of the
+    same algorithm (its decisions all with margin)."""
+    from paper_2305_10427_gb300 import ddgviz
+    from test_ddgviz import as_result
+    s = tiny_vary
+    checked = 0
+    for src in synth.sentences(25, 3, 6, 14, s.spec.vocab):
+        max_len = 2 * len(src)
+        s.dec.encode(src)
+        for m, b, rule in (("gs_jacobi", 5, "paper"), ("jacobi", 0, "suffix")):
+            r = s.dec.decode(m, max_len, b=b, trace=True, stop_rule=rule)
+            path = str(tmp_path / f"{m}.jsonl")
+            recs = ddgviz.dump_jsonl(r, path, method=m, b=b, stop_rule=rule, src=list(src))
+            assert ddgviz.load_jsonl(path) == recs
+            head, passes = recs[0], recs[1:]
+            assert head["tokens"] == r.tokens and head["n_passes"] == r.n_iters
+            for rec, row, tok in zip(passes, r.trace, r.trace_tokens):
+                assert rec["pass"] == row["step"] and rec["n_rows"] == row["n_rows"]
+                assert rec["tokens"] == list(tok[:row["block_len"]])
+            assert all(1 <= p <= r.n_iters for p in head["settled_at"])
+            ref = oracle_run(s.step(src), m, max_len, b, s.eos, rule)
+            if ref.min_margin > s.margin:
+                oh = ddgviz.trace_records(as_result(ref, max_len), method=m, b=b)[0]
+                assert oh["settled_at"] == head["settled_at"]
+                checked += 1
+    assert checked >= 2
