@@ -74,6 +74,7 @@ typedef struct {
   int max_batch;     /* capacity: sentences one pd_encode_batch / pd_decode_batch carries,
                         0 or 1..64 (0 = 1); each needs its own key/value caches */
   int gemm_engine;   /* pd_gemm_engine: how the bf16 matrix products run (fp32: always SIMT) */
+  int seed;          /* pd_create with weights = NULL: the seed of the drawn weights */
   int kv_pages;      /* capacity of each decoder layer's self-attention key/value pool, in
                         pages of 16 positions (0 = max_batch * ceil(max_tgt_len / 16)); a
                         decode needs sum over its sentences of ceil(max_len / 16) pages */
@@ -104,8 +105,13 @@ size_t pd_weights_nbytes(const pd_config* cfg);
 
 /* Create a context on the current CUDA device: validate cfg, allocate every device buffer for
  * the capacities in cfg, and upload the weight blob (host memory, nbytes =
- * pd_weights_nbytes(cfg)).  stream is a cudaStream_t (NULL: the library creates its own).
- * On success *out owns all device memory until pd_destroy. */
+ * pd_weights_nbytes(cfg)).  With weights = NULL and nbytes = 0 the library draws the weights
+ * itself from cfg->seed: element e of the blob's tensor number k (blob order, from 0) is
+ * 0.02 z, z the Box-Muller normal of the first two words of Philox-4x32-10 (Salmon et al., SC
+ * 2011) at counter (e / 2, k, 0, 0), key (seed, 0x5EED5EED) (cosine for even e, sine for odd),
+ * LayerNorm gains 1 and biases 0, rounded to the parameter type; pd_export_weights returns
+ * them.  stream is a cudaStream_t (NULL: the library creates its own).  On success *out owns
+ * all device memory until pd_destroy. */
 pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, void* stream,
                     pd_ctx** out);
 

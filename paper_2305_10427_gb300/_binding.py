@@ -48,7 +48,7 @@ class _Config(ctypes.Structure):
                                             "eos_id", "bos_id")] + \
               [("ln_eps", ctypes.c_float), ("max_src_len", ctypes.c_int),
                ("max_tgt_len", ctypes.c_int), ("max_batch", ctypes.c_int),
-               ("gemm_engine", ctypes.c_int), ("kv_pages", ctypes.c_int)]
+               ("gemm_engine", ctypes.c_int), ("seed", ctypes.c_int), ("kv_pages", ctypes.c_int)]
 
 
 class _DecodeParams(ctypes.Structure):
@@ -140,6 +140,7 @@ class Config:
     max_tgt_len: int = 256
     max_batch: int = 0
     gemm_engine: int = 0
+    seed: int = 0
     kv_pages: int = 0
 
     @classmethod
@@ -149,7 +150,7 @@ class Config:
         return cls(spec.d_model, spec.n_heads, spec.d_ff, spec.n_enc_layers, spec.n_dec_layers,
                    spec.vocab, spec.activation, bool(spec.pre_ln), bool(spec.learned_pos),
                    spec.max_pos, spec.dtype, pad_id, eos_id, bos_id, spec.ln_eps, max_src_len,
-                   max_tgt_len, max_batch, ENGINES[engine], kv_pages)
+                   max_tgt_len, max_batch, ENGINES[engine], 0, kv_pages)
 
     def _c(self) -> _Config:
         c = _Config()
@@ -180,19 +181,24 @@ def _i32p(a: np.ndarray):
 class Decoder:
     """One decoding context (pd_ctx) on the current CUDA device."""
 
-    def __init__(self, cfg: Config, weights: np.ndarray, stream: Optional[int] = None):
+    def __init__(self, cfg: Config, weights: Optional[np.ndarray], stream: Optional[int] = None):
+        """weights: the blob (host array), or None to have the library draw the weights from
+        cfg.seed."""
         self._lib = load_library()
         self.cfg = cfg
-        blob = np.ascontiguousarray(weights)
         self._ccfg = cfg._c()
         h = ctypes.c_void_p()
-        st = self._lib.pd_create(ctypes.byref(self._ccfg), blob.ctypes.data_as(ctypes.c_void_p),
-                                 blob.nbytes, ctypes.c_void_p(stream) if stream else None,
-                                 ctypes.byref(h))
+        if weights is None:
+            ptr, nbytes = None, 0
+        else:
+            blob = np.ascontiguousarray(weights)
+            ptr, nbytes = blob.ctypes.data_as(ctypes.c_void_p), blob.nbytes
+        st = self._lib.pd_create(ctypes.byref(self._ccfg), ptr, nbytes,
+                                 ctypes.c_void_p(stream) if stream else None, ctypes.byref(h))
         if st != PD_OK:
             raise PdError(st, "pd_create: " + self._lib.pd_last_error(None).decode())
         self._h = h
-        self.blob_nbytes = blob.nbytes
+        self.blob_nbytes = weights_nbytes(cfg)
 
     def _check(self, st: int, what: str):
         if st != PD_OK:

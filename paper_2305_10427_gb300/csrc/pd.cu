@@ -1019,6 +1019,26 @@ std::vector<std::pair<const W**, size_t>> layout(pd::ModelW<W>& mw, const pd_con
   return t;
 }
 
+// 1: the tensor is a LayerNorm gain, 2: a LayerNorm bias, 0: a weight or a linear bias.
+template <typename W>
+int ln_kind(const pd::ModelW<W>& mw, const W** field) {
+  const W* const* gains[] = {&mw.enc_lne_g, &mw.dec_lne_g, &mw.enc_lnf_g, &mw.dec_lnf_g};
+  const W* const* biases[] = {&mw.enc_lne_b, &mw.dec_lne_b, &mw.enc_lnf_b, &mw.dec_lnf_b};
+  for (auto g : gains) if (g == field) return 1;
+  for (auto b : biases) if (b == field) return 2;
+  for (int l = 0; l < pd::kMaxLayers; ++l) {
+    const auto& E = mw.enc[l];
+    const auto& L = mw.dec[l];
+    if (field == &E.ln1g || field == &E.ln2g || field == &L.ln1g || field == &L.ln2g ||
+        field == &L.ln3g)
+      return 1;
+    if (field == &E.ln1b || field == &E.ln2b || field == &L.ln1b || field == &L.ln2b ||
+        field == &L.ln3b)
+      return 2;
+  }
+  return 0;
+}
+
 size_t blob_elems(const pd_config& c) {
   pd::ModelW<float> mw{};
   size_t n = 0;
@@ -1163,9 +1183,18 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
   size_t soff = 0;
   for (size_t k = 0; k < lay.size(); ++k) {
     *lay[k].first = reinterpret_cast<const W*>(wdev + c->woff[k]);
-    PD_CUDA(c, cudaMemcpy(wdev + c->woff[k], src + soff, c->wbytes[k], cudaMemcpyHostToDevice));
+    if (src != nullptr) {
+      PD_CUDA(c, cudaMemcpy(wdev + c->woff[k], src + soff, c->wbytes[k], cudaMemcpyHostToDevice));
+    } else {                             // no blob: draw the weights from cfg.seed
+      pd::seeded_weights_kernel<W><<<c->n_sm * 4, 256, 0, c->stream>>>(
+          reinterpret_cast<W*>(wdev + c->woff[k]), lay[k].second, (unsigned)k,
+          (unsigned)cfg.seed, ln_kind(mw, lay[k].first), 0.02);
+      PD_CUDA(c, cudaGetLastError());
+      c->launches += 1;
+    }
     soff += c->wbytes[k];
   }
+  if (src == nullptr) PD_CUDA(c, cudaStreamSynchronize(c->stream));
   pd::ModelW<W>* mwd = nullptr;
   PD_TRY(dalloc(c, &mwd, 1));
   PD_CUDA(c, cudaMemcpy(mwd, &mw, sizeof(mw), cudaMemcpyHostToDevice));
@@ -1396,8 +1425,11 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   *out = nullptr;
   std::string why;
   if (!valid_config(cfg, &why)) { g_create_err = "invalid config: " + why; return PD_EINVAL; }
-  if (!weights) { g_create_err = "weights is NULL"; return PD_EINVAL; }
-  if (nbytes != pd_weights_nbytes(cfg)) {
+  if (!weights && nbytes != 0) {
+    g_create_err = "weights is NULL: nbytes must be 0 (the library draws the weights)";
+    return PD_EINVAL;
+  }
+  if (weights && nbytes != pd_weights_nbytes(cfg)) {
     g_create_err = "nbytes is " + std::to_string(nbytes) + ", the blob of this config has " +
                    std::to_string(pd_weights_nbytes(cfg));
     return PD_EINVAL;
@@ -1421,7 +1453,7 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   D.tc = cfg->dtype == PD_DTYPE_BF16 &&
          (cfg->gemm_engine == PD_ENGINE_TENSOR ||
           (cfg->gemm_engine == PD_ENGINE_AUTO && D.max_batch > 1));
-  c->blob_bytes = nbytes;
+  c->blob_bytes = pd_weights_nbytes(cfg);
   pd_status s = PD_OK;
   cudaError_t e = cudaGetDevice(&c->device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->n_sm, cudaDevAttrMultiProcessorCount, c->device);

@@ -253,6 +253,50 @@ __device__ __forceinline__ void l2_prefetch(const void* p, unsigned bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
+// Philox-4x32-10, the counter-based generator of Salmon, Moraes, Dror and Shaw ("Parallel
+// random numbers: as easy as 1, 2, 3", SC 2011): ten rounds of two 32x32 -> 64-bit multiplies
+// on a 4-word counter under a 2-word key bumped by the Weyl constants each round.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const unsigned long long p0 = 0xD2511F53ull * c.x, p1 = 0xCD9E8D57ull * c.z;
+    const unsigned hi0 = (unsigned)(p0 >> 32), lo0 = (unsigned)p0;
+    const unsigned hi1 = (unsigned)(p1 >> 32), lo1 = (unsigned)p1;
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+    k.x += 0x9E3779B9u;
+    k.y += 0xBB67AE85u;
+  }
+  return c;
+}
+
+// Seeded weights of tensor number `tensor` of the blob (kind 0: std * z, z standard normal;
+// 1: LayerNorm gain 1; 2: LayerNorm bias 0).  Element e draws Philox(counter (e / 2, tensor, 0,
+// 0), key (seed, 0x5EED5EED)); its first two words u1, u2 (as (x + 0.5) / 2^32) give by
+// Box-Muller z = sqrt(-2 ln u1) cos(2 pi u2) for even e, sin(2 pi u2) for odd e (in double
+// precision), then std * z rounded to the weight type.
+template <typename W>
+__global__ void seeded_weights_kernel(W* dst, size_t n, unsigned tensor, unsigned seed, int kind,
+                                      double std) {
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
+       e += (size_t)gridDim.x * blockDim.x) {
+    float v;
+    if (kind == 1) {
+      v = 1.0f;
+    } else if (kind == 2) {
+      v = 0.0f;
+    } else {
+      const uint4 r = philox4x32_10(make_uint4((unsigned)(e >> 1), tensor, 0u, 0u),
+                                    make_uint2(seed, 0x5EED5EEDu));
+      const double u1 = ((double)r.x + 0.5) * (1.0 / 4294967296.0);
+      const double u2 = ((double)r.y + 0.5) * (1.0 / 4294967296.0);
+      const double rad = sqrt(-2.0 * log(u1));
+      const double ang = 6.283185307179586476925286766559 * u2;
+      v = (float)(std * rad * ((e & 1) ? sin(ang) : cos(ang)));
+    }
+    dst[e] = from_f<W>(v);
+  }
+}
+
 // Sinusoidal position table, row p = [sin(p w_k) | cos(p w_k)], w_k = 10000^(-2k/d), in double
 // precision rounded to fp32 (run once when a context is created).
 __global__ void sinusoid_kernel(float* tab, int rows, int d) {
