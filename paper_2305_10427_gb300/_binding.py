@@ -145,12 +145,13 @@ class Config:
 
     @classmethod
     def from_spec(cls, spec, max_src_len: int, max_tgt_len: int, pad_id=1, eos_id=0, bos_id=2,
-                  max_batch: int = 0, engine: str = "auto", kv_pages: int = 0):
-        """Build from any object carrying the model fields (d_model, n_heads, ...)."""
+                  max_batch: int = 0, engine: str = "auto", kv_pages: int = 0, seed: int = 0):
+        """Build from any object carrying the model fields (d_model, n_heads, ...); seed is
+        used only when the Decoder is created without a weight blob."""
         return cls(spec.d_model, spec.n_heads, spec.d_ff, spec.n_enc_layers, spec.n_dec_layers,
                    spec.vocab, spec.activation, bool(spec.pre_ln), bool(spec.learned_pos),
                    spec.max_pos, spec.dtype, pad_id, eos_id, bos_id, spec.ln_eps, max_src_len,
-                   max_tgt_len, max_batch, ENGINES[engine], 0, kv_pages)
+                   max_tgt_len, max_batch, ENGINES[engine], seed, kv_pages)
 
     def _c(self) -> _Config:
         c = _Config()

@@ -94,9 +94,7 @@ def gpu():
 
 
 def _drawn(pkg, spec, seed, **kw):
-    import dataclasses
-    cfg = dataclasses.replace(pkg.Config.from_spec(spec, 32, 32, **kw), seed=seed)
-    return pkg.Decoder(cfg, None)
+    return pkg.Decoder(pkg.Config.from_spec(spec, 32, 32, seed=seed, **kw), None)
 
 
 @pytest.mark.gpu
