@@ -31,7 +31,8 @@ import synth  # noqa: E402
 
 WORKLOAD = synth.MARIAN_GS
 STOP_RULE = "paper"          # "paper": StopC of Eq. 5; "prefix": accepted-prefix rule
-ENGINE = "auto"              # pd_gemm_engine: auto (SIMT at batch 1, tensor cores batched)
+ENGINE = "auto"              # pd_gemm_engine (auto = SIMT)
+CLUSTER_SIZE = 0             # cluster engine: CTAs per cluster (0 = the library's choice)
 ARGS_WORKLOAD = "marian"
 METRIC = "translated tokens/s at batch 1, GS-Jacobi vs greedy AR; HBM GB/s % of peak"
 FALLBACK_HBM_GBS = 6800.0
@@ -269,7 +270,8 @@ def run_gpu(args):
     max_src = max(len(s) for s in sents)
     max_tgt = max(WORKLOAD.max_len(len(s)) for s in sents)
     stream = torch.cuda.Stream()
-    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, engine=ENGINE), weights.blob,
+    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, engine=ENGINE,
+                                           cluster_size=CLUSTER_SIZE), weights.blob,
                       stream=stream.cuda_stream)
 
     offs = np.cumsum([0] + [len(s) for s in sents])
@@ -407,7 +409,7 @@ def run_gpu(args):
             "data": "synthetic: seeded N(0,0.02) weights, uniform random source ids",
             "config": {"workload": WORKLOAD.name if n_s == WORKLOAD.n_sentences else
                        f"{WORKLOAD.name} (first {n_s} sentences only)", "sentences_per_step": n_s,
-                       "stop_rule": STOP_RULE, "engine": ENGINE,
+                       "stop_rule": STOP_RULE, "engine": ENGINE, "cluster_size": CLUSTER_SIZE,
                        "timing": "CUDA events on the library stream; L2 flushed (256 MB write) "
                                  "between steps; replicas across GPUs"},
             "greedy": {"value": greedy_tps, "unit": "tokens/s",
@@ -463,7 +465,8 @@ def run_gpu_batch(args):
     max_src = max(len(s) for s in sents)
     max_tgt = max(WORKLOAD.max_len(len(s)) for s in sents)
     stream = torch.cuda.Stream()
-    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, max_batch=S, engine=ENGINE),
+    dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, max_batch=S, engine=ENGINE,
+                                           cluster_size=CLUSTER_SIZE),
                       weights.blob, stream=stream.cuda_stream)
     offs_all = np.cumsum([0] + [len(s) for s in sents])
     d_src = torch.tensor(np.concatenate(sents), dtype=torch.int32, device="cuda")
@@ -538,7 +541,8 @@ def run_gpu_batch(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic: seeded N(0,0.02) weights, uniform random source ids",
             "config": {"workload": f"{WORKLOAD.name}, batches of {S} sentences",
-                       "sentences_per_step": len(sents), "batch": S, "stop_rule": STOP_RULE, "engine": ENGINE,
+                       "sentences_per_step": len(sents), "batch": S, "stop_rule": STOP_RULE,
+                       "engine": ENGINE, "cluster_size": CLUSTER_SIZE,
                        "timing": "CUDA events on the library stream around encode + decode of "
                                  "all batches; L2 flushed (256 MB write) between steps"},
             "greedy": {"value": greedy_tps, "unit": "tokens/s",
@@ -581,16 +585,19 @@ def main():
                          "or one pass per position); prefix = also once the unchanged leading "
                          "tokens make the whole block exact")
     ap.add_argument("--oracle-worker", action="store_true", help=argparse.SUPPRESS)
-    ap.add_argument("--engine", default="auto", choices=["auto", "simt", "tensor"],
-                    help="matrix-product engine of the bf16 context (pd_gemm_engine)")
+    ap.add_argument("--engine", default="auto", choices=["auto", "simt", "tensor", "cluster"],
+                    help="decoder engine of the context (pd_gemm_engine)")
+    ap.add_argument("--cluster-size", type=int, default=0, choices=[0, 2, 4, 8],
+                    help="cluster engine: CTAs per thread-block cluster (0 = the library's)")
     ap.add_argument("--batch", type=int, default=1,
                     help="sentences decoded together (batched serving); 1 = the batch-1 benchmark")
     ap.add_argument("--sentences", type=int, default=0,
                     help="use only the first N sentences of the workload (profiling runs)")
     args = ap.parse_args()
-    global WORKLOAD, STOP_RULE, ENGINE, ARGS_WORKLOAD
+    global WORKLOAD, STOP_RULE, ENGINE, ARGS_WORKLOAD, CLUSTER_SIZE
     STOP_RULE = args.stop_rule
     ENGINE = args.engine
+    CLUSTER_SIZE = args.cluster_size
     ARGS_WORKLOAD = args.workload
     if args.workload == "marian-knob":
         WORKLOAD = synth.MARIAN_KNOB

@@ -73,24 +73,34 @@ typedef struct {
   int max_tgt_len;   /* capacity: largest max_len pd_decode accepts */
   int max_batch;     /* capacity: sentences one pd_encode_batch / pd_decode_batch carries,
                         0 or 1..64 (0 = 1); each needs its own key/value caches */
-  int gemm_engine;   /* pd_gemm_engine: how the bf16 matrix products run (fp32: always SIMT) */
+  int gemm_engine;   /* pd_gemm_engine: how the decoder passes run (fp32: SIMT or CLUSTER) */
   int seed;          /* pd_create with weights = NULL: the seed of the drawn weights */
   int kv_pages;      /* capacity of each decoder layer's self-attention key/value pool, in
                         pages of 16 positions (0 = max_batch * ceil(max_tgt_len / 16)); a
                         decode needs sum over its sentences of ceil(max_len / 16) pages */
+  int cluster_size;  /* PD_ENGINE_CLUSTER: CTAs per thread-block cluster, 2, 4 or 8 (0 = 8) */
 } pd_config;
 
-/* How a bf16 context runs the matrix products of its encoder and decoder passes.  Every pass of
- * a context uses the same engine, so each row's arithmetic is the same whatever the pass
- * carries and every decoding method returns exactly the context's greedy tokens; the two
- * engines round differently (both within the bf16 parity bar).
- *  PD_ENGINE_SIMT: CUDA-core dot products spread over every SM; the latency-bound choice for
- *    passes of a few rows (one sentence, small blocks).
- *  PD_ENGINE_TENSOR: 5th-generation tensor cores (tcgen05, accumulators in tensor memory),
- *    weight tiles streamed by TMA; the choice when passes carry many rows (batched serving,
- *    full-sentence Jacobi).
- *  PD_ENGINE_AUTO: TENSOR when max_batch > 1, else SIMT. */
-typedef enum { PD_ENGINE_AUTO = 0, PD_ENGINE_SIMT = 1, PD_ENGINE_TENSOR = 2 } pd_gemm_engine;
+/* How a context runs its decoder passes (and the matrix products of its encoder).  Every pass
+ * of a context uses the same engine, so each row's arithmetic is the same whatever the pass
+ * carries and every decoding method returns exactly the context's greedy tokens; the engines
+ * round differently (all within the parity bar).
+ *  PD_ENGINE_SIMT: CUDA-core dot products spread over every SM, the 8 steps of a decoder layer
+ *    separated by grid barriers.
+ *  PD_ENGINE_TENSOR (bf16 only): the SIMT engine's phases with every matrix product on the
+ *    5th-generation tensor cores (tcgen05, accumulators in tensor memory), weight tiles
+ *    streamed by TMA.
+ *  PD_ENGINE_CLUSTER: a decoder layer as three super-phases (self-attention, cross-attention,
+ *    FFN), each run per attention head or per slice of FFN hidden units by a thread-block
+ *    cluster of cluster_size CTAs that exchange rows through distributed shared memory, with
+ *    one grid barrier per super-phase; CUDA-core products, SIMT encoder.
+ *  PD_ENGINE_AUTO: SIMT. */
+typedef enum {
+  PD_ENGINE_AUTO = 0,
+  PD_ENGINE_SIMT = 1,
+  PD_ENGINE_TENSOR = 2,
+  PD_ENGINE_CLUSTER = 3
+} pd_gemm_engine;
 
 typedef struct pd_ctx pd_ctx;
 

@@ -25,7 +25,7 @@ METHODS = {"greedy": 0, "jacobi": 1, "gs_jacobi": 2, "hybrid_gs_jacobi": 3}
 STOP_RULES = {"paper": 0, "prefix": 1, "suffix": 2}   # pd_stop_rule: Eq. 5 StopC, accepted
 #                                                     prefix, accepted prefix with suffix re-runs
 INITS = {"pad": 0, "last": 1}                         # pd_init_rule
-ENGINES = {"auto": 0, "simt": 1, "tensor": 2}   # pd_gemm_engine
+ENGINES = {"auto": 0, "simt": 1, "tensor": 2, "cluster": 3}   # pd_gemm_engine
 
 # Every symbol include/pd.h declares.
 EXPORTED = ("pd_weights_nbytes", "pd_create", "pd_export_weights", "pd_encode",
@@ -48,7 +48,8 @@ class _Config(ctypes.Structure):
                                             "eos_id", "bos_id")] + \
               [("ln_eps", ctypes.c_float), ("max_src_len", ctypes.c_int),
                ("max_tgt_len", ctypes.c_int), ("max_batch", ctypes.c_int),
-               ("gemm_engine", ctypes.c_int), ("seed", ctypes.c_int), ("kv_pages", ctypes.c_int)]
+               ("gemm_engine", ctypes.c_int), ("seed", ctypes.c_int), ("kv_pages", ctypes.c_int),
+               ("cluster_size", ctypes.c_int)]
 
 
 class _DecodeParams(ctypes.Structure):
@@ -142,16 +143,19 @@ class Config:
     gemm_engine: int = 0
     seed: int = 0
     kv_pages: int = 0
+    cluster_size: int = 0
 
     @classmethod
     def from_spec(cls, spec, max_src_len: int, max_tgt_len: int, pad_id=1, eos_id=0, bos_id=2,
-                  max_batch: int = 0, engine: str = "auto", kv_pages: int = 0, seed: int = 0):
+                  max_batch: int = 0, engine: str = "auto", kv_pages: int = 0, seed: int = 0,
+                  cluster_size: int = 0):
         """Build from any object carrying the model fields (d_model, n_heads, ...); seed is
-        used only when the Decoder is created without a weight blob."""
+        used only when the Decoder is created without a weight blob, cluster_size only by the
+        cluster engine."""
         return cls(spec.d_model, spec.n_heads, spec.d_ff, spec.n_enc_layers, spec.n_dec_layers,
                    spec.vocab, spec.activation, bool(spec.pre_ln), bool(spec.learned_pos),
                    spec.max_pos, spec.dtype, pad_id, eos_id, bos_id, spec.ln_eps, max_src_len,
-                   max_tgt_len, max_batch, ENGINES[engine], seed, kv_pages)
+                   max_tgt_len, max_batch, ENGINES[engine], seed, kv_pages, cluster_size)
 
     def _c(self) -> _Config:
         c = _Config()

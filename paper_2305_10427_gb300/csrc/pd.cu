@@ -24,6 +24,7 @@
 #include "pd.h"
 #include "pd_device.cuh"
 #include "tc_gemm.cuh"
+#include "cl_pass.cuh"
 
 namespace pd {
 
@@ -60,6 +61,11 @@ struct SmemLayout {
   // total includes the 1024 bytes of alignment slack
   size_t ring, bbuf, epi;
   int ring_slots;
+  // cluster-engine kernels (cl_pass.cuh): xs holds the staged fp32 rows of a tile; us the
+  // sublayer inputs, qs the tile's scaled queries, as its attention outputs, hs its FFN hidden
+  // units (part holds the products' warp sums and the LM head's partials; scratch the
+  // attention scores and warp sums)
+  size_t us, qs, as, hs;
 };
 
 // The commit region: per pass row r (at most D.rows) its new token (-1 for a NaN row) and
@@ -144,6 +150,24 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
     const size_t all = vec_smem_bytes(D, wsize), ln = ln_elems(D) * wsize;
     L.ln_bytes = L.ln + all <= budget ? all : (L.ln + ln <= budget && ln <= kVecSmemMax ? ln : 0);
     L.total = 1024 + L.ln + L.ln_bytes;
+    return L;
+  }
+  if (D.cl) {
+    auto a16 = [](size_t b) { return (b + 15) / 16 * 16; };
+    L.xs = 0;
+    L.us = L.xs + a16((size_t)kClRows * D.d * 4);
+    L.qs = L.us + a16((size_t)kClRows * D.d * wsize);
+    L.as = L.qs + a16((size_t)kClRows * D.dh * 4);
+    L.hs = L.as + a16((size_t)kClRows * D.dh * wsize);
+    L.part = L.hs + a16((size_t)kClRows * D.cl_fu * D.cl * wsize);
+    L.scratch = L.part + (size_t)kWarps * 32 * sizeof(Partial);
+    L.commit = L.scratch + a16(((size_t)D.max_keys + 2 * kWarps + (size_t)kWarps * D.dh) * 4);
+    L.ln = a16(L.commit + commit_bytes(D));
+    const size_t all = vec_smem_bytes(D, wsize), ln = ln_elems(D) * wsize;
+    const size_t slack = wsize == 2 ? 1024 : 0;   // smem_base's alignment of bf16 kernels
+    L.ln_bytes = L.ln + all + slack <= kSmemMax ? all
+                 : (L.ln + ln + slack <= kSmemMax && ln <= kVecSmemMax ? ln : 0);
+    L.total = slack + L.ln + L.ln_bytes;
     return L;
   }
   const int kmax = D.d > D.f ? D.d : D.f;
@@ -508,6 +532,241 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
   return true;
 }
 
+// Shared-memory regions and pass-wide values of the cluster engine's super-phases, kept in
+// shared memory (like the GEMM arguments of the SIMT engine) so that the products' loops do
+// not hold them in registers.
+template <typename W>
+struct ClCtx {
+  float* ys;
+  W* us;
+  float* qs;
+  W* as;
+  W* hs;
+  float* red;
+  float* sc;
+  float* wred;
+  int rank, cid, ncl, u, nffn;
+  size_t part_ld;
+  CommitMem cm;
+};
+template <typename W>
+__device__ __forceinline__ ClCtx<W>& smem_clctx() {
+  __shared__ ClCtx<W> s;
+  return s;
+}
+template <typename W>
+__device__ __forceinline__ ClGemm<W>& smem_clgemm() {
+  __shared__ ClGemm<W> s;
+  return s;
+}
+template <typename W>
+__device__ __forceinline__ ClStage<W>& smem_clstage() {
+  __shared__ ClStage<W> s;
+  return s;
+}
+// Thread 0, once per kernel.
+template <typename W>
+__device__ void cl_ctx_init(unsigned char* smem) {
+  const Dims& D = smem_dims<W>();
+  const SmemLayout SL = smem_layout(D, sizeof(W));
+  ClCtx<W>& c = smem_clctx<W>();
+  c.ys = reinterpret_cast<float*>(smem + SL.xs);
+  c.us = reinterpret_cast<W*>(smem + SL.us);
+  c.qs = reinterpret_cast<float*>(smem + SL.qs);
+  c.as = reinterpret_cast<W*>(smem + SL.as);
+  c.hs = reinterpret_cast<W*>(smem + SL.hs);
+  c.red = reinterpret_cast<float*>(smem + SL.part);
+  c.sc = reinterpret_cast<float*>(smem + SL.scratch);
+  c.wred = c.sc + D.max_keys;
+  c.rank = (int)cl_rank();
+  c.cid = (int)cl_index();
+  c.ncl = (int)cl_count();
+  c.u = D.cl_fu * D.cl;
+  c.nffn = (D.f + c.u - 1) / c.u;
+  c.part_ld = (size_t)D.rows * D.d;
+  c.cm = commit_mem(D, smem + SL.commit);
+}
+
+// A product of the cluster engine: thread 0 fills the shared argument block (fill(g) on a
+// cleared block), the CTA runs it, and meets again before the block can be refilled.
+template <typename W, bool SHORT = false, typename F>
+__device__ __forceinline__ void cl_product(F&& fill) {
+  ClGemm<W>& g = smem_clgemm<W>();
+  if (threadIdx.x == 0) {
+    g = ClGemm<W>{};
+    fill(g);
+  }
+  __syncthreads();
+  cl_gemm<W, SHORT>(g, smem_clctx<W>().red);
+  __syncthreads();
+}
+
+// Super-phase SA (self) or SB (cross) of layer l for the heads of this cluster: per tile of
+// rows, stage, then per head the queries (and self keys / values), attention, and the head's
+// share of the output projection into partial sum h of p_out.
+template <typename W>
+__device__ __noinline__ void cl_attn_super(const KParams<W>& P, int l, bool self, int M,
+                                           float* p_out) {
+  const Dims& D = smem_dims<W>();
+  const ClCtx<W>& c = smem_clctx<W>();
+  const int dh = D.dh, cs = D.cl;
+  for (int m0 = 0; m0 < M; m0 += kClRows) {
+    const int mt = M - m0 < kClRows ? M - m0 : kClRows;
+    cl_stage(smem_clstage<W>(), smem_tabs<W>(), D, c.cm.rtok, c.cm.rpos, m0, mt, c.ys, c.us,
+             c.red);
+    for (int h = c.cid; h < D.H; h += c.ncl) {
+      const size_t self_ld = (size_t)D.kv_pages * kPageRows * D.d;
+      const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
+      // queries (and, self-attention, the keys / values of the tile's rows) of head h
+      cl_product<W>([&](ClGemm<W>& g) {
+        const DecLayerW<W>& L = smem_mw<W>().dec[l];
+        g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d; g.dh = dh;
+        g.K = D.d; g.xs = c.us; g.ldx = D.d; g.hoff = h * dh; g.qs = c.qs;
+        g.scale = 1.0f / sqrtf((float)dh);
+        if (self) {
+          g.N = 3 * dh; g.wr = ClRows<W>{L.wqkv, D.d, h * dh, dh, D.d, 0};
+          g.epi = CL_QKV; g.bias = L.bqkv; g.slot = c.cm.rslot;
+          g.kdst = P.B.kself + l * self_ld; g.vdst = P.B.vself + l * self_ld;
+        } else {
+          g.N = dh; g.wr = ClRows<W>{L.wqc, D.d, h * dh, dh, 0, 0};
+          g.epi = CL_Q; g.bias = L.bqc + h * dh;
+        }
+      });
+      cl_sync();
+      // attention of the tile's rows (rows rank, rank + cs, ... of this CTA)
+      for (int r = c.rank; r < mt; r += cs) {
+        const int m = m0 + r;
+        if (self)
+          cl_attn_row<W>(D, c.qs + r * dh, P.B.kself + l * self_ld, P.B.vself + l * self_ld,
+                         h * dh, c.cm.rkn[m], c.cm.pt, c.cm.rsb[m], c.sc, c.wred, c.as + r * dh);
+        else
+          cl_attn_row<W>(D, c.qs + r * dh, P.B.kcross + l * cross_ld, P.B.vcross + l * cross_ld,
+                         h * dh, c.cm.rxn[m], nullptr, c.cm.rxb[m], c.sc, c.wred, c.as + r * dh);
+      }
+      cl_sync();
+      // head h's share of the output projection: partial sum h
+      cl_product<W, true>([&](ClGemm<W>& g) {
+        const DecLayerW<W>& L = smem_mw<W>().dec[l];
+        g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d; g.dh = dh;
+        g.N = D.d; g.K = dh; g.wr = ClRows<W>{self ? L.wo : L.woc, D.d, 0, D.d, 0, h * dh};
+        g.xs = c.as; g.ldx = dh; g.epi = CL_PART; g.gout = p_out + (size_t)h * c.part_ld;
+      });
+    }
+  }
+}
+
+// Super-phase SC of layer l for this cluster's FFN hidden units: per tile of rows, stage,
+// FFN1 of the units with the activation into every CTA's hs, and the units' share of FFN2 into
+// partial sum cid of p_out.
+template <typename W>
+__device__ __noinline__ void cl_ffn_super(const KParams<W>& P, int l, int M, float* p_out) {
+  const Dims& D = smem_dims<W>();
+  const ClCtx<W>& c = smem_clctx<W>();
+  const int cs = D.cl;
+  const int c0 = c.cid * c.u, nc = D.f - c0 < c.u ? D.f - c0 : c.u;
+  for (int m0 = 0; m0 < M; m0 += kClRows) {
+    const int mt = M - m0 < kClRows ? M - m0 : kClRows;
+    cl_stage(smem_clstage<W>(), smem_tabs<W>(), D, c.cm.rtok, c.cm.rpos, m0, mt, c.ys, c.us,
+             c.red);
+    cl_product<W>([&](ClGemm<W>& g) {
+      const DecLayerW<W>& L = smem_mw<W>().dec[l];
+      g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d;
+      g.N = nc; g.K = D.d; g.wr = ClRows<W>{L.w1, D.d, c0, nc, 0, 0}; g.xs = c.us; g.ldx = D.d;
+      g.epi = CL_HID; g.bias = L.b1 + c0; g.hs = c.hs; g.ldh = c.u; g.act = D.act;
+    });
+    cl_sync();
+    cl_product<W, true>([&](ClGemm<W>& g) {
+      const DecLayerW<W>& L = smem_mw<W>().dec[l];
+      g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d;
+      g.N = D.d; g.K = nc; g.wr = ClRows<W>{L.w2, D.f, 0, D.d, 0, c0}; g.xs = c.hs; g.ldx = c.u;
+      g.epi = CL_PART; g.gout = p_out + (size_t)c.cid * c.part_ld;
+    });
+  }
+}
+
+// The LM head over the whole grid: every cluster stages the final rows for its CTAs; argmax
+// partials per CTA and row (or raw logits).
+template <typename W>
+__device__ __noinline__ void cl_lm_super(const KParams<W>& P, int M, float* logits) {
+  const Dims& D = smem_dims<W>();
+  const ClCtx<W>& c = smem_clctx<W>();
+  for (int m0 = 0; m0 < M; m0 += kClRows) {
+    const int mt = M - m0 < kClRows ? M - m0 : kClRows;
+    cl_stage(smem_clstage<W>(), smem_tabs<W>(), D, c.cm.rtok, c.cm.rpos, m0, mt, c.ys, c.us,
+             c.red);
+    cl_product<W>([&](ClGemm<W>& g) {
+      g.m0 = m0; g.mt = mt; g.d = D.d;
+      g.N = D.V; g.K = D.d; g.wr = ClRows<W>{smem_mw<W>().embed, D.d, 0, D.V, 0, 0};
+      g.xs = c.us; g.ldx = D.d; g.nct = (int)gridDim.x; g.cta = (int)blockIdx.x; g.ncl = D.cl;
+      g.epi = logits != nullptr ? CL_LOGITS : CL_ARGMAX;
+      g.logits = logits; g.part = P.B.part; g.part_ld = D.rows;
+    });
+  }
+}
+
+// One decoder pass of the cluster engine (cl_pass.cuh) over the M rows described in the
+// commit region: per layer the super-phases SA (self-attention), SB (cross-attention) and SC
+// (FFN), each followed by a grid barrier, then the LM head.  Super-phase s reads the residual
+// rows R[s & 1] and the partial sums P[s & 1] the previous one left, and writes R[(s+1) & 1]
+// (cluster 0) and P[(s+1) & 1]; the two sets alternate, so no super-phase overwrites what
+// another cluster may still be reading.  False if a barrier gave up.
+template <typename W>
+__device__ bool run_pass_cl(const KParams<W>& P, int M, float* logits, unsigned& tgt,
+                            unsigned char* smem) {
+  const Dims& D = smem_dims<W>();
+  const Bufs<W>& B = P.B;
+  const ModelW<W>& mw = smem_mw<W>();
+  const bool pre = D.pre_ln != 0;
+  const int cid = (int)cl_index();
+  const int u = D.cl_fu * D.cl, nffn = (D.f + u - 1) / u;
+  const size_t part_ld = (size_t)D.rows * D.d;
+  if (threadIdx.x == 0) cl_ctx_init<W>(smem);
+  prefetch_gemm_weights(mw.embed, D.V, D.d);       // the LM head's table, asked from L2 early
+  for (int s = 0;; ++s) {
+    const int l = s / 3, kind = s - 3 * l;        // kind 0 SA, 1 SB, 2 SC; s = 3 Ld: LM head
+    const bool lm = s == 3 * D.Ld;
+    float* p_out = B.clp + ((s & 1) ? 0 : (size_t)D.cl_np * part_ld);
+    if (threadIdx.x == 0) {
+      ClStage<W>& st = smem_clstage<W>();
+      st = ClStage<W>{};
+      st.r_in = (s & 1) ? B.rb : B.ra;
+      st.part = B.clp + ((s & 1) ? (size_t)D.cl_np * part_ld : 0);
+      st.part_ld = part_ld;
+      st.r_out = lm ? nullptr : ((s & 1) ? B.ra : B.rb);
+      if (s == 0) {                               // layer 0 starts from the embedding
+        st.emb = 1;
+        if (pre) { st.lna_g = mw.dec_lne_g; st.lna_b = mw.dec_lne_b; }
+      } else {                                    // what the previous super-phase left
+        const int pk = (s - 1) % 3;
+        const DecLayerW<W>& PL = mw.dec[(s - 1) / 3];
+        st.np = pk == 2 ? nffn : D.H;
+        st.bias = pk == 0 ? PL.bo : (pk == 1 ? PL.boc : PL.b2);
+        if (!pre) {                               // post-LN: the sublayer's LayerNorm
+          st.lna_g = pk == 0 ? PL.ln1g : (pk == 1 ? PL.ln2g : PL.ln3g);
+          st.lna_b = pk == 0 ? PL.ln1b : (pk == 1 ? PL.ln2b : PL.ln3b);
+        }
+      }
+      if (pre) {                                  // pre-LN: this sublayer's input LayerNorm
+        if (lm) {
+          st.lnb_g = mw.dec_lnf_g; st.lnb_b = mw.dec_lnf_b;
+        } else {
+          const DecLayerW<W>& L = mw.dec[l];
+          st.lnb_g = kind == 0 ? L.ln1g : (kind == 1 ? L.ln2g : L.ln3g);
+          st.lnb_b = kind == 0 ? L.ln1b : (kind == 1 ? L.ln2b : L.ln3b);
+        }
+      }
+    }
+    __syncthreads();
+    if (lm) {
+      cl_lm_super<W>(P, M, logits);
+      return true;                                // the caller's barrier follows
+    }
+    if (kind < 2 && cid < D.H) cl_attn_super<W>(P, l, kind == 0, M, p_out);
+    else if (kind == 2 && cid < nffn) cl_ffn_super<W>(P, l, M, p_out);
+    if (!cl_grid_barrier(B.bar, tgt, &B.st->status)) return false;
+  }
+}
+
 // ------------------------------------------------------------------------------------------
 // fixed-point commit (every CTA): StopC of Eq. 5, block advance of Algorithms 1-3, trace row
 // ------------------------------------------------------------------------------------------
@@ -731,7 +990,7 @@ __device__ void write_outputs(const KParams<W>& P, unsigned char* smem) {
 // kernels
 // ------------------------------------------------------------------------------------------
 
-template <typename W, bool TC>
+template <typename W, bool TC, bool CL = false>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ KParams<W> P) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   unsigned char* smem = smem_base<W>(smem_raw);
@@ -755,7 +1014,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
       cm.rxb[m] = 0; cm.rxn[m] = P.n_src_s[0];
     }
     __syncthreads();
-    run_pass<W, TC>(P, P.debug_len, P.logits, tgt, smem, false);
+    if constexpr (CL) {
+      run_pass_cl<W>(P, P.debug_len, P.logits, tgt, smem);
+      cl_sync();                          // no CTA leaves while a partner may read its memory
+    } else {
+      run_pass<W, TC>(P, P.debug_len, P.logits, tgt, smem, false);
+    }
     if constexpr (TC) tc_teardown<W>();
     return;
   }
@@ -784,12 +1048,18 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   for (;;) {
     const int M = cm.misc[0];
     if (M == 0) break;
-    if (!run_pass<W, TC>(P, M, nullptr, tgt, smem, true)) break;
-    if (!grid_barrier(B.bar, tgt, status, [&] { stream_weights<W, TC>(P, smem); })) break;
+    if constexpr (CL) {
+      if (!run_pass_cl<W>(P, M, nullptr, tgt, smem)) break;
+      if (!cl_grid_barrier(B.bar, tgt, status)) break;
+    } else {
+      if (!run_pass<W, TC>(P, M, nullptr, tgt, smem, true)) break;
+      if (!grid_barrier(B.bar, tgt, status, [&] { stream_weights<W, TC>(P, smem); })) break;
+    }
     commit<W>(P, smem);
   }
   if (blockIdx.x == 0) write_outputs(P, smem);
   if constexpr (TC) tc_teardown<W>();
+  if constexpr (CL) cl_sync();
 }
 
 // The encoder pass of encode_kernel: every encoder layer (QKV, full self-attention, O, FFN1,
@@ -916,6 +1186,7 @@ struct pd_ctx {
   cudaStream_t stream = nullptr;
   bool own_stream = false;
   int device = 0, n_sm = 0, grid = 0;
+  int cl_grid = 0;                            // cluster engine: CTAs of the decode grid
   size_t smem = 0;
   std::vector<void*> allocs;
   void* wdev = nullptr;                       // device weights (tensors 256-byte aligned)
@@ -972,7 +1243,11 @@ bool valid_config(const pd_config* c, std::string* why) {
     if (id < 0 || id >= c->vocab) return bad("special ids must be in [0, vocab)");
   if (!(c->ln_eps >= 0.f)) return bad("ln_eps");
   if (c->max_batch < 0 || c->max_batch > pd::kMaxBatch) return bad("max_batch must be in [0, 64]");
-  if (c->gemm_engine < PD_ENGINE_AUTO || c->gemm_engine > PD_ENGINE_TENSOR) return bad("gemm_engine");
+  if (c->gemm_engine < PD_ENGINE_AUTO || c->gemm_engine > PD_ENGINE_CLUSTER) return bad("gemm_engine");
+  if (c->gemm_engine == PD_ENGINE_TENSOR && c->dtype != PD_DTYPE_BF16)
+    return bad("the tensor-core engine needs bf16 weights");
+  if (c->cluster_size != 0 && c->cluster_size != 2 && c->cluster_size != 4 && c->cluster_size != 8)
+    return bad("cluster_size must be 0, 2, 4 or 8");
   if (c->kv_pages != 0 &&
       (c->kv_pages < (c->max_tgt_len + pd::kPageRows - 1) / pd::kPageRows || c->kv_pages > (1 << 20)))
     return bad("kv_pages must be 0 or hold one sentence of max_tgt_len (<= 2^20 pages)");
@@ -1067,13 +1342,15 @@ pd_status dalloc(pd_ctx* c, T** p, size_t count) {
     if (s_ != PD_OK) return s_;    \
   } while (0)
 
-// The decode / encode kernel of a context's engine (bf16 only has the tensor-core one).
+// The decode / encode kernel of a context's engine (bf16 only has the tensor-core one; the
+// cluster engine's encoder is the SIMT one).
 template <typename W>
-const void* kernel_fn(bool encode, bool tc) {
+const void* kernel_fn(bool encode, bool tc, bool cl = false) {
   if constexpr (sizeof(W) == 2) {
     if (tc) return encode ? (const void*)pd::encode_kernel<W, true>
                           : (const void*)pd::decode_kernel<W, true>;
   }
+  if (cl && !encode) return (const void*)pd::decode_kernel<W, false, true>;
   return encode ? (const void*)pd::encode_kernel<W, false> : (const void*)pd::decode_kernel<W, false>;
 }
 
@@ -1163,6 +1440,57 @@ pd_status tc_resources(pd_ctx* c, const pd::ModelW<__nv_bfloat16>& mw) {
   return PD_OK;
 }
 
+// Cluster-engine geometry of a context: as many clusters of D.cl CTAs as can be resident at
+// once with the decode kernel's shared memory (at most n_sm / D.cl), FFN hidden units per CTA
+// so that the clusters cover d_ff, and the partial-sum buffers ([2][max(H, FFN slices)][rows]
+// [d] fp32).  The FFN share and the shared memory depend on each other, so the two are
+// settled together.
+template <typename W>
+pd_status cl_resources(pd_ctx* c) {
+  Dims& D = c->D;
+  const void* fdec = kernel_fn<W>(false, false, true);
+  Dims De = D;
+  De.cl = 0;
+  const size_t smem_enc = pd::smem_layout(De, sizeof(W)).total;   // the (SIMT) encoder's
+  int ncl = c->n_sm / D.cl;
+  for (int it = 0;; ++it) {
+    D.cl_n = ncl;
+    // units per cluster: a multiple of 16, so that every slice starts on a 16-byte boundary
+    // of the FFN2 rows and holds whole 16-byte chunks
+    const int per = (D.f + ncl - 1) / ncl, u = (per + 15) / 16 * 16, nffn = (D.f + u - 1) / u;
+    D.cl_fu = u / D.cl;
+    D.cl_np = std::max(D.H, nffn);
+    const size_t smem = std::max(pd::smem_layout(D, sizeof(W)).total, smem_enc);
+    if (smem > pd::kSmemMax)
+      return fail(c, PD_EINVAL, "the cluster engine's shared memory does not fit (max_tgt_len "
+                                "or max_batch too large)");
+    cudaFuncAttributes a{};
+    PD_CUDA(c, cudaFuncGetAttributes(&a, fdec));
+    if ((size_t)a.maxDynamicSharedSizeBytes < smem)
+      PD_CUDA(c, cudaFuncSetAttribute(fdec, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    cudaLaunchConfig_t lc{};
+    lc.gridDim = dim3(ncl * D.cl);
+    lc.blockDim = dim3(pd::kThreads);
+    lc.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = (unsigned)D.cl;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    int fit = 0;
+    PD_CUDA(c, cudaOccupancyMaxActiveClusters(&fit, fdec, &lc));
+    if (fit >= ncl) break;
+    if (fit < 1 || it >= 8) return fail(c, PD_EINVAL, "no cluster of the decode kernel fits an SM group");
+    ncl = fit;
+  }
+  c->cl_grid = D.cl_n * D.cl;
+  pd::Bufs<W>& B = bufs<W>(c);
+  PD_TRY(dalloc(c, &B.clp, 2 * (size_t)D.cl_np * D.rows * D.d));
+  return PD_OK;
+}
+
 template <typename W>
 pd_status create_impl(pd_ctx* c, const void* weights) {
   const pd_config& cfg = c->cfg;
@@ -1238,12 +1566,18 @@ pd_status create_impl(pd_ctx* c, const void* weights) {
     if (D.tc) PD_TRY(tc_resources(c, mw));
   }
 
+  if (D.cl) PD_TRY(cl_resources<W>(c));
   c->smem = pd::smem_layout(D, sizeof(W)).total;
+  if (D.cl) {                                 // the encoder runs the SIMT layout
+    Dims De = D;
+    De.cl = 0;
+    c->smem = std::max(c->smem, pd::smem_layout(De, sizeof(W)).total);
+  }
   if (D.tc && pd::smem_layout(D, sizeof(W)).ring_slots < 2)
     return fail(c, PD_EINVAL, "the tensor-core kernels' shared memory does not fit (max_tgt_len "
                               "or max_batch too large)");
   // the limit is per kernel function and shared by every context of the process: only raise it
-  const void* fdec = kernel_fn<W>(false, D.tc != 0);
+  const void* fdec = kernel_fn<W>(false, D.tc != 0, D.cl != 0);
   const void* fenc = kernel_fn<W>(true, D.tc != 0);
   PD_TRY(raise_smem_limit(c, fdec));
   PD_TRY(raise_smem_limit(c, fenc));
@@ -1276,7 +1610,27 @@ pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P, bool reset_status = 
     std::memcpy(P.maps, maps.data(), maps.size() * sizeof(CUtensorMap));
   }
   void* args[] = {&P};
-  const void* fn = kernel_fn<W>(encode, c->D.tc != 0);
+  const void* fn = kernel_fn<W>(encode, c->D.tc != 0, c->D.cl != 0);
+  if (c->D.cl && !encode) {                   // clusters of D.cl CTAs, cooperative (co-resident)
+    cudaLaunchConfig_t lc{};
+    lc.gridDim = dim3(c->cl_grid);
+    lc.blockDim = dim3(pd::kThreads);
+    lc.dynamicSmemBytes = c->smem;
+    lc.stream = c->stream;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = (unsigned)c->D.cl;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeCooperative;
+    at[1].val.cooperative = 1;
+    lc.attrs = at;
+    lc.numAttrs = 2;
+    PD_CUDA(c, cudaLaunchKernelExC(&lc, fn, args));
+    c->launches += 1;
+    return PD_OK;
+  }
+  if (encode) P.D.cl = 0;                     // the cluster engine's encoder is the SIMT one
   PD_CUDA(c, cudaLaunchCooperativeKernel(fn, dim3(c->grid), dim3(pd::kThreads), args, c->smem,
                                          c->stream));
   c->launches += 1;
@@ -1450,9 +1804,8 @@ pd_status pd_create(const pd_config* cfg, const void* weights, size_t nbytes, vo
   D.kv_pages = cfg->kv_pages > 0 ? cfg->kv_pages : D.max_batch * D.pt_ld;
   const long batch_rows = std::min<long>((long)D.max_batch * D.max_tgt, pd::kMaxPassRows);
   D.rows = (int)std::max<long>(D.max_keys, batch_rows);
-  D.tc = cfg->dtype == PD_DTYPE_BF16 &&
-         (cfg->gemm_engine == PD_ENGINE_TENSOR ||
-          (cfg->gemm_engine == PD_ENGINE_AUTO && D.max_batch > 1));
+  D.tc = cfg->dtype == PD_DTYPE_BF16 && cfg->gemm_engine == PD_ENGINE_TENSOR;
+  D.cl = cfg->gemm_engine == PD_ENGINE_CLUSTER ? (cfg->cluster_size > 0 ? cfg->cluster_size : 8) : 0;
   c->blob_bytes = pd_weights_nbytes(cfg);
   pd_status s = PD_OK;
   cudaError_t e = cudaGetDevice(&c->device);

@@ -72,6 +72,10 @@ struct Dims {
   int tc;          // bf16: GEMM phases on the tensor cores (else the SIMT path)
   int kv_pages;    // pages of kPageRows cache rows in each decoder layer's self K/V pool
   int pt_ld;       // page-table entries per sentence: ceil(max_tgt / kPageRows)
+  int cl;          // cluster engine (cl_pass.cuh): decoder passes as per-layer super-phases
+  int cl_n;        // cluster engine: clusters of the decode grid
+  int cl_fu;       // cluster engine: FFN hidden units per CTA (cl_fu * kCl per cluster)
+  int cl_np;       // cluster engine: partial sums a super-phase can leave (max(H, FFN slices))
 };
 
 // Per-CTA partial of the LM-head argmax for one row.
@@ -120,6 +124,7 @@ struct Bufs {
                                // page (written by the host before a decode)
   float* red;                  // bf16: split-K partial sums [S][rows][N]
   unsigned* cnt;               // bf16: split-K arrival counters (zero between uses)
+  float* clp;                  // cluster engine: partial sums [2][cl_np][rows][d]
 };
 
 // ------------------------------------------------------------------------------------------

@@ -139,6 +139,7 @@ def test_binding_enums_match_header():
                                                   "PD_INIT_LAST": B.INITS["last"]}
     assert _enum_values(text, "pd_gemm_engine") == {"PD_ENGINE_AUTO": B.ENGINES["auto"],
                                                     "PD_ENGINE_SIMT": B.ENGINES["simt"],
-                                                    "PD_ENGINE_TENSOR": B.ENGINES["tensor"]}
+                                                    "PD_ENGINE_TENSOR": B.ENGINES["tensor"],
+                                                    "PD_ENGINE_CLUSTER": B.ENGINES["cluster"]}
     status = _enum_values(text, "pd_status")
     assert {v: k for k, v in status.items()} == B.STATUS_NAMES

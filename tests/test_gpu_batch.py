@@ -32,9 +32,9 @@ def _gpu():
     torch.cuda.set_device(0)
 
 
-def _decoder(spec, max_batch, eos=synth.EOS_ID, **wkw):
+def _decoder(spec, max_batch, eos=synth.EOS_ID, engine="auto", **wkw):
     w = synth.make_weights(spec, **wkw)
-    cfg = pkg.Config.from_spec(spec, 64, 128, eos_id=eos, max_batch=max_batch)
+    cfg = pkg.Config.from_spec(spec, 64, 128, eos_id=eos, max_batch=max_batch, engine=engine)
     return w, pkg.Decoder(cfg, w.blob)
 
 
@@ -44,12 +44,15 @@ MODELS = {
     "tiny_eos": (synth.TINY, 3038, dict(seed=5, embed_std=0.005)),
     "marian": (synth.MARIAN, synth.EOS_ID, dict(seed=0)),
 }
+# (model, engine) pairs of the batch-versus-single test
+BATCH_CASES = [(m, "simt") for m in MODELS] + [("marian", "tensor"), ("tiny_vary", "cluster"),
+                                               ("tiny_eos", "cluster"), ("marian", "cluster")]
 
 
-@pytest.mark.parametrize("name", list(MODELS))
-def test_batch_equals_single(name):
+@pytest.mark.parametrize("name,engine", BATCH_CASES)
+def test_batch_equals_single(name, engine):
     spec, eos, kw = MODELS[name]
-    _, dec = _decoder(spec, 4, eos=eos, **kw)
+    _, dec = _decoder(spec, 4, eos=eos, engine=engine, **kw)
     sents = synth.sentences(61, 4, 5, 20, spec.vocab)
     max_len = [2 * len(s) for s in sents]
     single = {}
@@ -127,7 +130,7 @@ def test_batch_errors():
     dec.close()
 
 
-@pytest.mark.parametrize("engine", ["simt", "tensor"])
+@pytest.mark.parametrize("engine", ["simt", "tensor", "cluster"])
 def test_paged_cache_pool(engine):
     """The self-attention keys and values live in a pool of 16-position pages handed out per
     decode (sentence s's pages interleaved with the others', never contiguous in a batch).  A
@@ -135,7 +138,7 @@ def test_paged_cache_pool(engine):
     would need) decodes every sentence exactly as a context with the default pool decodes it
     alone, and a request that needs more pages than the pool holds is rejected before any
     launch."""
-    spec = synth.TINY if engine == "simt" else MODELS["marian"][0]
+    spec = MODELS["marian"][0] if engine == "tensor" else synth.TINY
     w = synth.make_weights(spec, seed=0)
     big = pkg.Decoder(pkg.Config.from_spec(spec, 64, 128, engine=engine), w.blob)
     small = pkg.Decoder(pkg.Config.from_spec(spec, 64, 128, max_batch=4, engine=engine,

@@ -54,14 +54,16 @@ def _gpu():
 
 
 class Setup:
-    def __init__(self, spec, max_src, max_tgt, eos=synth.EOS_ID, engine="auto", **wkw):
+    def __init__(self, spec, max_src, max_tgt, eos=synth.EOS_ID, engine="auto", cluster_size=0,
+                 **wkw):
         self.spec = spec
         self.eos = eos
         self.margin = MARGIN_BF16 if spec.dtype == synth.DTYPE_BF16 else MARGIN_F32
         self.w = synth.make_weights(spec, **wkw)
         self.model = om.Model(spec, self.w.tensors)
         self.dec = pkg.Decoder(pkg.Config.from_spec(spec, max_src, max_tgt, eos_id=eos,
-                                                    engine=engine), self.w.blob)
+                                                    engine=engine, cluster_size=cluster_size),
+                               self.w.blob)
         self._mem = {}
 
     def mem(self, src):
@@ -98,6 +100,14 @@ def tiny():
 
 
 @pytest.fixture(scope="module")
+def tiny_cl():
+    """The tiny model on the cluster engine (PD_ENGINE_CLUSTER)."""
+    s = Setup(synth.TINY, 64, 64, engine="cluster", seed=0)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
 def tiny_ln():
     """Tiny model with perturbed LayerNorm gains and biases, so that every parameter counts."""
     s = Setup(synth.TINY, 64, 64, seed=3, ln_noise=0.2)
@@ -110,6 +120,13 @@ def tiny_vary():
     """Tiny model with a small token-embedding scale: its outputs change along the sentence
     and Jacobi converges in fewer than m passes."""
     s = Setup(synth.TINY, 64, 64, seed=5, embed_std=0.005)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
+def tiny_vary_cl():
+    s = Setup(synth.TINY, 64, 64, engine="cluster", seed=5, embed_std=0.005)
     yield s
     s.dec.close()
 
@@ -164,6 +181,22 @@ def bf16_knob_tc():
 
 
 @pytest.fixture(scope="module")
+def bf16_knob_cl():
+    s = _bf16_knob("cluster")
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
+def bf16_knob_cl4():
+    """The cluster engine with clusters of 4 CTAs."""
+    s = Setup(BF16_KNOB, 64, 128, engine="cluster", cluster_size=4, seed=12, ln_noise=1.0,
+              embed_std=0.012)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
 def marian():
     s = Setup(synth.MARIAN, 64, 128, engine="simt", seed=0)
     yield s
@@ -173,6 +206,13 @@ def marian():
 @pytest.fixture(scope="module")
 def marian_tc():
     s = Setup(synth.MARIAN, 64, 128, engine="tensor", seed=0)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
+def marian_cl():
+    s = Setup(synth.MARIAN, 64, 128, engine="cluster", seed=0)
     yield s
     s.dec.close()
 
@@ -287,7 +327,7 @@ def test_export_roundtrip(tiny, marian):
 
 # ---- logits --------------------------------------------------------------------------------
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_ln"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_ln", "tiny_cl"])
 def test_tiny_logits_fp32(name, request):
     s = request.getfixturevalue(name)
     rng = np.random.default_rng(11)
@@ -300,7 +340,7 @@ def test_tiny_logits_fp32(name, request):
         assert rel_row_err(got, ref).max() < 1e-4
 
 
-@pytest.mark.parametrize("name", ["marian", "marian_tc"])
+@pytest.mark.parametrize("name", ["marian", "marian_tc", "marian_cl"])
 def test_marian_logits_bf16(name, request):
     s = request.getfixturevalue(name)
     rng = np.random.default_rng(12)
@@ -313,7 +353,8 @@ def test_marian_logits_bf16(name, request):
         assert rel_row_err(got, ref).max() < 2e-2
 
 
-@pytest.mark.parametrize("name", ["tiny", "bf16_knob", "bf16_knob_tc", "marian", "marian_tc"])
+@pytest.mark.parametrize("name", ["tiny", "bf16_knob", "bf16_knob_tc", "marian", "marian_tc",
+                                  "tiny_cl", "bf16_knob_cl", "bf16_knob_cl4", "marian_cl"])
 def test_logits_batch_invariant(name, request):
     """Batch invariance, the property behind every method's bit identity with greedy: the
     logits of row t (inputs y_0..y_t) are the same bits whether the pass carries t + 1 rows or
@@ -332,7 +373,8 @@ def test_logits_batch_invariant(name, request):
 
 # ---- tokens, bit identity, traces ------------------------------------------------------------
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_ln", "tiny_vary", "tiny_eos"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_ln", "tiny_vary", "tiny_eos", "tiny_cl",
+                                  "tiny_vary_cl"])
 def test_tiny_all_methods(name, request):
     s = request.getfixturevalue(name)
     srcs = [synth.TINY_JACOBI.sentences()[0]] + synth.sentences(21, 3, 5, 30, s.spec.vocab)
@@ -362,7 +404,7 @@ def oracle_run(step, method, max_len, b, eos, rule, init_rule="pad"):
 
 
 @pytest.mark.parametrize("name", ["tiny_vary", "tiny_eos", "tiny_fast", "bf16_knob",
-                                  "bf16_knob_tc"])
+                                  "bf16_knob_tc", "tiny_vary_cl", "bf16_knob_cl"])
 def test_suffix_rule_and_last_token_init(name, request):
     """Options the paper leaves to future work (Section 5): the suffix-only re-run (same
     passes and trace as the accepted-prefix rule, fewer rows: n_rows in the trace) and the
@@ -455,7 +497,7 @@ def test_tiny_eos_paths(tiny_eos):
     assert seen_eos >= 2
 
 
-@pytest.mark.parametrize("name", ["bf16_knob", "bf16_knob_tc"])
+@pytest.mark.parametrize("name", ["bf16_knob", "bf16_knob_tc", "bf16_knob_cl", "bf16_knob_cl4"])
 def test_bf16_traces_against_oracle(name, request):
     """bf16 weights: pass counts, per-pass traces and DDGviz probabilities of every method equal
     the oracle's step-by-step runs (all of its decisions clear the bf16 margin), and blocks
@@ -477,7 +519,7 @@ def test_bf16_traces_against_oracle(name, request):
 
 
 @pytest.mark.parametrize("name", ["tiny", "tiny_vary", "bf16_knob", "bf16_knob_tc", "marian",
-                                  "marian_tc"])
+                                  "marian_tc", "tiny_cl", "bf16_knob_cl", "marian_cl"])
 def test_trace_probs_against_own_logits_and_oracle(name, request):
     """The DDGviz probability of each greedy pass (softmax probability of the argmax, Section
     3.5) is computed on the device by an online sum of exponentials merged across CTA partials.
@@ -505,7 +547,7 @@ def test_trace_probs_against_own_logits_and_oracle(name, request):
         assert (err <= 2 * dl + LOGP_SLACK).all(), err.max()
 
 
-@pytest.mark.parametrize("name", ["marian", "marian_tc"])
+@pytest.mark.parametrize("name", ["marian", "marian_tc", "marian_cl"])
 def test_marian_methods_bit_identical(name, request):
     marian = request.getfixturevalue(name)
     for src in synth.sentences(41, 3, 8, 12, marian.spec.vocab):
@@ -528,7 +570,7 @@ def test_marian_methods_bit_identical(name, request):
         assert frac >= MARIAN_MIN_COVERED
 
 
-@pytest.mark.parametrize("name", ["marian", "marian_tc"])
+@pytest.mark.parametrize("name", ["marian", "marian_tc", "marian_cl"])
 def test_marian_full_size_sampled(name, request):
     """The benchmark's launch configuration (GS-Jacobi b=5, max_len = 2n) on the longest
     sentence lengths of the workload: tokens checked by one teacher-forced oracle pass."""
@@ -680,13 +722,28 @@ def pre_bf16():
 
 
 @pytest.fixture(scope="module")
+def pre_f32_cl():
+    s = Setup(PRE_F32, 64, 64, engine="cluster", seed=11, ln_noise=0.2, embed_std=0.05)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
+def pre_bf16_cl():
+    s = Setup(PRE_BF16, 64, 64, engine="cluster", seed=12, ln_noise=0.2, embed_std=0.05)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
 def pre_bf16_tc():
     s = Setup(PRE_BF16, 64, 64, engine="tensor", seed=12, ln_noise=0.2, embed_std=0.05)
     yield s
     s.dec.close()
 
 
-@pytest.mark.parametrize("name", ["pre_f32", "pre_bf16", "pre_bf16_tc"])
+@pytest.mark.parametrize("name", ["pre_f32", "pre_bf16", "pre_bf16_tc", "pre_f32_cl",
+                                  "pre_bf16_cl"])
 def test_pre_ln_models(name, request):
     """Pre-LN blocks with embedding and final LayerNorms, exact GELU and a learned position
     table: logits against the oracle, every method bit-identical to the GPU's greedy, pass
@@ -711,7 +768,7 @@ def test_pre_ln_models(name, request):
     assert compared >= 3
 
 
-@pytest.mark.parametrize("engine", ["simt", "tensor"])
+@pytest.mark.parametrize("engine", ["simt", "tensor", "cluster"])
 def test_mbart_full_size_sampled(engine):
     """The mBART-large-sized preset at its full size (d = 1024, 12 + 12 layers, d_ff = 4096,
     V = 250027, pre-LN, GELU, learned positions): teacher-forced logits of a few rows against
