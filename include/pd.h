@@ -78,7 +78,8 @@ typedef struct {
   int kv_pages;      /* capacity of each decoder layer's self-attention key/value pool, in
                         pages of 16 positions (0 = max_batch * ceil(max_tgt_len / 16)); a
                         decode needs sum over its sentences of ceil(max_len / 16) pages */
-  int cluster_size;  /* PD_ENGINE_CLUSTER: CTAs per thread-block cluster, 2, 4 or 8 (0 = 8) */
+  int cluster_size;  /* PD_ENGINE_CLUSTER: CTAs per thread-block cluster, 1, 2, 4 or 8 (0 = 8;
+                        1 = a plain cooperative launch, every CTA a cluster of one) */
 } pd_config;
 
 /* How a context runs its decoder passes (and the matrix products of its encoder).  Every pass

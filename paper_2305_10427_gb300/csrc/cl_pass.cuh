@@ -155,19 +155,19 @@ __device__ __forceinline__ float cl_dot(const W* w0, int ldw, int nvalid, int j0
       wr[c] = c < nvalid ? ldg_nc_v4(w0 + (size_t)c * ldw + (size_t)j * E)
                          : make_uint4(0u, 0u, 0u, 0u);
     if constexpr (sizeof(W) == 2) {
+      float wv[kNCol][8];
 #pragma unroll
-      for (int c = 0; c < kNCol; ++c) {
-        float wv[8];
-        unpack8(wr[c], wv);
+      for (int c = 0; c < kNCol; ++c) unpack8(wr[c], wv[c]);
 #pragma unroll
-        for (int r = 0; r < kMTile; ++r) {
-          if (r < mt) {
-            float x[8];
-            unpack8(*reinterpret_cast<const uint4*>(xs + (size_t)r * ldx + (size_t)j * E), x);
+      for (int r = 0; r < kMTile; ++r) {
+        if (r < mt) {
+          float x[8];
+          unpack8(*reinterpret_cast<const uint4*>(xs + (size_t)r * ldx + (size_t)j * E), x);
+#pragma unroll
+          for (int c = 0; c < kNCol; ++c)
 #pragma unroll
             for (int e = 0; e < 8; ++e)
-              acc[c * kMTile + r] = fmaf(wv[e], x[e], acc[c * kMTile + r]);
-          }
+              acc[c * kMTile + r] = fmaf(wv[c][e], x[e], acc[c * kMTile + r]);
         }
       }
     } else {
@@ -273,33 +273,37 @@ struct ClGemm {
 };
 
 // Outputs (n, r), n < N, r < mt, of sum_k wr.row(n)[k] * xs[r][k], k < K, by nct CTAs (this one
-// is cta): group g of outputs 4g..4g+3 goes to CTA g mod nct and, within it, to warp slot
-// (g / nct) mod gpc; its K chunks are split into kw contiguous ranges, one per warp, whose
-// sums are added in warp order.  Every thread of the CTA calls this.  red: [kWarps][32] floats
-// (or Partials for CL_ARGMAX) of shared memory.
-template <typename W, bool SHORT>
+// is cta), with epilogue EPI (a compile-time choice, so each call site carries only its own):
+// group g of outputs 4g..4g+3 goes to CTA g mod nct and, within it, to warp slot (g / nct) mod
+// gpc; its K chunks are split into kw contiguous ranges, one per warp, whose sums are added in
+// warp order.  Every thread of the CTA calls this.  red: [kWarps][32] floats and as many ints
+// (or [kWarps][32] Partials for CL_ARGMAX) of shared memory.
+template <typename W, int EPI, bool SHORT>
 __device__ __forceinline__ void cl_gemm(const ClGemm<W>& g, float* red) {
   constexpr int E = 16 / (int)sizeof(W);
+  constexpr bool argmax = EPI == CL_ARGMAX;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int ngroups = (g.N + kNCol - 1) / kNCol, nch = g.K / E;
-  constexpr bool shortk = SHORT;          // one lane per output (K of at most 32 chunks)
-  const int kw = shortk ? 1 : cl_kw(ngroups, nch, g.nct);
+  int ngroups, nch, kw, nct, cta, N, mt;
+  {
+    N = g.N; mt = g.mt; nct = g.nct; cta = g.cta;
+    ngroups = (N + kNCol - 1) / kNCol;
+    nch = g.K / E;
+    kw = SHORT ? 1 : cl_kw(ngroups, nch, nct);
+  }
   const int gpc = kWarps / kw;
   const int slot = warp / kw, part = warp - slot * kw;
   const int j0 = part * nch / kw, j1 = (part + 1) * nch / kw;
-  const int c = lane / kMTile, r = lane % kMTile;
-  const int mt = g.mt;
   float amx = -INFINITY, asum = 0.f;
   int aidx = 0x7fffffff, anan = 0;
-  for (int base = 0; base < ngroups; base += g.nct * gpc) {
-    const int gi = base + slot * g.nct + g.cta;
+  for (int base = 0; base < ngroups; base += nct * gpc) {
+    const int gi = base + slot * nct + cta;
     const bool active = slot < gpc && gi < ngroups;
     const int n0 = gi * kNCol;
-    const int nvalid = active ? (g.N - n0 < kNCol ? g.N - n0 : kNCol) : 0;
+    const int nvalid = active ? (N - n0 < kNCol ? N - n0 : kNCol) : 0;
     float a = 0.f;
     if (active)
-      a = shortk ? cl_dot_short<W>(g.wr.row(n0), g.wr.ldw, nvalid, nch, g.xs, g.ldx, mt)
-                 : cl_dot<W>(g.wr.row(n0), g.wr.ldw, nvalid, j0, j1, g.xs, g.ldx, mt);
+      a = SHORT ? cl_dot_short<W>(g.wr.row(n0), g.wr.ldw, nvalid, nch, g.xs, g.ldx, mt)
+                : cl_dot<W>(g.wr.row(n0), g.wr.ldw, nvalid, j0, j1, g.xs, g.ldx, mt);
     if (kw > 1) {
       if (active) red[warp * 32 + lane] = a;
       __syncthreads();
@@ -307,29 +311,48 @@ __device__ __forceinline__ void cl_gemm(const ClGemm<W>& g, float* red) {
         for (int q = 1; q < kw; ++q) a += red[(warp + q) * 32 + lane];
       __syncthreads();
     }
-    if (!active || part != 0 || r >= mt || c >= nvalid) continue;
-    const int n = n0 + c, m = g.m0 + r;
-    float v = a;
-    switch (g.epi) {
-      case CL_QKV: {
-        const int w = n / g.dh, e = n - w * g.dh;
-        v += to_f(g.bias[w * g.d + g.hoff + e]);
-        if (w == 0) {
-          cl_bcast(g.qs + r * g.dh + e, v * g.scale, g.ncl);
-        } else {
-          W* dst = (w == 1 ? g.kdst : g.vdst) + (size_t)g.slot[m] * g.d + g.hoff + e;
-          *dst = from_f<W>(v);
+    const int c = lane / kMTile, r = lane % kMTile;
+    const bool valid = active && part == 0 && r < mt && c < nvalid;
+    if constexpr (argmax) {
+      if (valid) argmax_push(a, n0 + c, amx, aidx, asum, anan);
+    } else {
+      // the epilogue runs after a barrier, one thread per value of this round, reading its
+      // arguments from shared memory there (nothing of it stays live across the products)
+      int* okf = reinterpret_cast<int*>(red + kWarps * 32);
+      red[warp * 32 + lane] = a;
+      okf[warp * 32 + lane] = valid;
+      __syncthreads();
+      {
+        const int w2 = threadIdx.x >> 5, l2 = threadIdx.x & 31;
+        const float v0 = red[threadIdx.x];
+        const int s2 = w2 / kw;
+        const int n = (base + s2 * nct + cta) * kNCol + l2 / kMTile, m = g.m0 + l2 % kMTile;
+        if (okf[threadIdx.x]) {
+          float v = v0;
+          if constexpr (EPI == CL_QKV) {
+            const int w = n / g.dh, e = n - w * g.dh;
+            v += to_f(g.bias[w * g.d + g.hoff + e]);
+            if (w == 0) {
+              cl_bcast(g.qs + (l2 % kMTile) * g.dh + e, v * g.scale, g.ncl);
+            } else {
+              W* dst = (w == 1 ? g.kdst : g.vdst) + (size_t)g.slot[m] * g.d + g.hoff + e;
+              *dst = from_f<W>(v);
+            }
+          } else if constexpr (EPI == CL_Q) {
+            cl_bcast(g.qs + (l2 % kMTile) * g.dh + n, (v + to_f(g.bias[n])) * g.scale, g.ncl);
+          } else if constexpr (EPI == CL_PART) {
+            g.gout[(size_t)m * g.d + n] = v;
+          } else if constexpr (EPI == CL_HID) {
+            cl_bcast(g.hs + (l2 % kMTile) * g.ldh + n, act_fn(v + to_f(g.bias[n]), g.act), g.ncl);
+          } else if constexpr (EPI == CL_LOGITS) {
+            g.logits[(size_t)m * g.N + n] = v;
+          }
         }
-        break;
       }
-      case CL_Q: cl_bcast(g.qs + r * g.dh + n, (v + to_f(g.bias[n])) * g.scale, g.ncl); break;
-      case CL_PART: g.gout[(size_t)m * g.d + n] = v; break;
-      case CL_HID: cl_bcast(g.hs + r * g.ldh + n, act_fn(v + to_f(g.bias[n]), g.act), g.ncl); break;
-      case CL_LOGITS: g.logits[(size_t)m * g.N + n] = v; break;
-      case CL_ARGMAX: argmax_push(v, n, amx, aidx, asum, anan); break;
+      __syncthreads();
     }
   }
-  if (g.epi == CL_ARGMAX) {
+  if constexpr (argmax) {
     // lane c*8 + r holds row r over its columns 4g + c; a row's partials are merged in
     // (warp, column) order, then by a fixed butterfly (as gemm_phase)
     Partial* ps = reinterpret_cast<Partial*>(red);
@@ -440,33 +463,20 @@ __device__ __forceinline__ void cl_stage_sum(const ClStage<W>& a, const Dims& D,
   }
 }
 
-// LayerNorm of the row y[0..d) (shared memory, fp32) by one warp, in place: mean and biased
-// variance from per-lane sums over elements lane * 4 + 128 i (ascending i), fixed butterflies.
+// LayerNorm of the row y[0..d) (shared memory, fp32) by one warp, in place (ln_regs: mean and
+// biased variance from per-lane sums over elements lane * 4 + 128 i, fixed butterflies).
 template <typename W>
 __device__ __forceinline__ void cl_ln_row(float* y, int d, const W* g, const W* b, float eps) {
   const int lane = threadIdx.x & 31;
-  float s = 0.f;
-  for (int k = lane * 4; k < d; k += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(y + k);
-    s += (v.x + v.y) + (v.z + v.w);
-  }
-  const float mean = warp_sum(s) / d;
-  float s2 = 0.f;
-  for (int k = lane * 4; k < d; k += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(y + k);
-    const float a0 = v.x - mean, a1 = v.y - mean, a2 = v.z - mean, a3 = v.w - mean;
-    s2 += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
-  }
-  const float rstd = 1.0f / sqrtf(warp_sum(s2) / d + eps);
-  for (int k = lane * 4; k < d; k += 128) {
-    float4 v = *reinterpret_cast<const float4*>(y + k);
-    const float4 gk = get4(g + k), bk = get4(b + k);
-    v.x = (v.x - mean) * rstd * gk.x + bk.x;
-    v.y = (v.y - mean) * rstd * gk.y + bk.y;
-    v.z = (v.z - mean) * rstd * gk.z + bk.z;
-    v.w = (v.w - mean) * rstd * gk.w + bk.w;
-    *reinterpret_cast<float4*>(y + k) = v;
-  }
+  const int nI = d / 128;
+  float4 v[kMaxRowRegs];
+#pragma unroll
+  for (int i = 0; i < kMaxRowRegs; ++i)
+    if (i < nI) v[i] = *reinterpret_cast<const float4*>(y + lane * 4 + 128 * i);
+  ln_regs(v, nI, d, g, b, eps);
+#pragma unroll
+  for (int i = 0; i < kMaxRowRegs; ++i)
+    if (i < nI) *reinterpret_cast<float4*>(y + lane * 4 + 128 * i) = v[i];
   __syncwarp();
 }
 

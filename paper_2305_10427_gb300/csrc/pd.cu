@@ -589,7 +589,7 @@ __device__ void cl_ctx_init(unsigned char* smem) {
 
 // A product of the cluster engine: thread 0 fills the shared argument block (fill(g) on a
 // cleared block), the CTA runs it, and meets again before the block can be refilled.
-template <typename W, bool SHORT = false, typename F>
+template <typename W, int EPI, bool SHORT = false, typename F>
 __device__ __forceinline__ void cl_product(F&& fill) {
   ClGemm<W>& g = smem_clgemm<W>();
   if (threadIdx.x == 0) {
@@ -597,7 +597,7 @@ __device__ __forceinline__ void cl_product(F&& fill) {
     fill(g);
   }
   __syncthreads();
-  cl_gemm<W, SHORT>(g, smem_clctx<W>().red);
+  cl_gemm<W, EPI, SHORT>(g, smem_clctx<W>().red);
   __syncthreads();
 }
 
@@ -618,7 +618,7 @@ __device__ __noinline__ void cl_attn_super(const KParams<W>& P, int l, bool self
       const size_t self_ld = (size_t)D.kv_pages * kPageRows * D.d;
       const size_t cross_ld = (size_t)D.max_batch * D.max_src * D.d;
       // queries (and, self-attention, the keys / values of the tile's rows) of head h
-      cl_product<W>([&](ClGemm<W>& g) {
+      auto fill_q = [&](ClGemm<W>& g) {
         const DecLayerW<W>& L = smem_mw<W>().dec[l];
         g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d; g.dh = dh;
         g.K = D.d; g.xs = c.us; g.ldx = D.d; g.hoff = h * dh; g.qs = c.qs;
@@ -631,7 +631,9 @@ __device__ __noinline__ void cl_attn_super(const KParams<W>& P, int l, bool self
           g.N = dh; g.wr = ClRows<W>{L.wqc, D.d, h * dh, dh, 0, 0};
           g.epi = CL_Q; g.bias = L.bqc + h * dh;
         }
-      });
+      };
+      if (self) cl_product<W, CL_QKV>(fill_q);
+      else cl_product<W, CL_Q>(fill_q);
       cl_sync();
       // attention of the tile's rows (rows rank, rank + cs, ... of this CTA)
       for (int r = c.rank; r < mt; r += cs) {
@@ -645,7 +647,7 @@ __device__ __noinline__ void cl_attn_super(const KParams<W>& P, int l, bool self
       }
       cl_sync();
       // head h's share of the output projection: partial sum h
-      cl_product<W, true>([&](ClGemm<W>& g) {
+      cl_product<W, CL_PART, true>([&](ClGemm<W>& g) {
         const DecLayerW<W>& L = smem_mw<W>().dec[l];
         g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d; g.dh = dh;
         g.N = D.d; g.K = dh; g.wr = ClRows<W>{self ? L.wo : L.woc, D.d, 0, D.d, 0, h * dh};
@@ -668,14 +670,14 @@ __device__ __noinline__ void cl_ffn_super(const KParams<W>& P, int l, int M, flo
     const int mt = M - m0 < kClRows ? M - m0 : kClRows;
     cl_stage(smem_clstage<W>(), smem_tabs<W>(), D, c.cm.rtok, c.cm.rpos, m0, mt, c.ys, c.us,
              c.red);
-    cl_product<W>([&](ClGemm<W>& g) {
+    cl_product<W, CL_HID>([&](ClGemm<W>& g) {
       const DecLayerW<W>& L = smem_mw<W>().dec[l];
       g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d;
       g.N = nc; g.K = D.d; g.wr = ClRows<W>{L.w1, D.d, c0, nc, 0, 0}; g.xs = c.us; g.ldx = D.d;
       g.epi = CL_HID; g.bias = L.b1 + c0; g.hs = c.hs; g.ldh = c.u; g.act = D.act;
     });
     cl_sync();
-    cl_product<W, true>([&](ClGemm<W>& g) {
+    cl_product<W, CL_PART, true>([&](ClGemm<W>& g) {
       const DecLayerW<W>& L = smem_mw<W>().dec[l];
       g.m0 = m0; g.mt = mt; g.nct = cs; g.cta = c.rank; g.ncl = cs; g.d = D.d;
       g.N = D.d; g.K = nc; g.wr = ClRows<W>{L.w2, D.f, 0, D.d, 0, c0}; g.xs = c.hs; g.ldx = c.u;
@@ -694,13 +696,52 @@ __device__ __noinline__ void cl_lm_super(const KParams<W>& P, int M, float* logi
     const int mt = M - m0 < kClRows ? M - m0 : kClRows;
     cl_stage(smem_clstage<W>(), smem_tabs<W>(), D, c.cm.rtok, c.cm.rpos, m0, mt, c.ys, c.us,
              c.red);
-    cl_product<W>([&](ClGemm<W>& g) {
+    auto fill = [&](ClGemm<W>& g) {
       g.m0 = m0; g.mt = mt; g.d = D.d;
       g.N = D.V; g.K = D.d; g.wr = ClRows<W>{smem_mw<W>().embed, D.d, 0, D.V, 0, 0};
       g.xs = c.us; g.ldx = D.d; g.nct = (int)gridDim.x; g.cta = (int)blockIdx.x; g.ncl = D.cl;
       g.epi = logits != nullptr ? CL_LOGITS : CL_ARGMAX;
       g.logits = logits; g.part = P.B.part; g.part_ld = D.rows;
-    });
+    };
+    if (logits != nullptr) cl_product<W, CL_LOGITS>(fill);
+    else cl_product<W, CL_ARGMAX>(fill);
+  }
+}
+
+// Ask L2 for the weight rows this CTA reads in super-phase s (row segments of its product
+// groups: group g of a product goes to CTA g mod cs of the cluster), while it waits at the grid
+// barrier before it.
+template <typename W>
+__device__ void cl_prefetch(int s, int tid, int nthreads) {
+  const Dims& D = smem_dims<W>();
+  const ClCtx<W>& c = smem_clctx<W>();
+  if (s >= 3 * D.Ld) return;                     // the LM head's table is asked at pass start
+  const int l = s / 3, kind = s - 3 * l, cs = D.cl, dh = D.dh;
+  const DecLayerW<W>& L = smem_mw<W>().dec[l];
+  // rows of product (wr, N, K) that this CTA's groups read (group g of 4 rows goes to CTA
+  // g mod cs), one 16-byte aligned segment each; this thread takes rows tid, tid + nthreads, ...
+  // of the CTA's list, numbered on from t
+  auto rows = [&](const ClRows<W>& wr, int N, int K, int& t) {
+    const int ng = (N + kNCol - 1) / kNCol;
+    const int mine = ng > c.rank ? (ng - c.rank + cs - 1) / cs : 0;   // groups of this CTA
+    const int nr = mine * kNCol;
+    for (int i = ((tid - t) % nthreads + nthreads) % nthreads; i < nr; i += nthreads) {
+      const int n = (c.rank + (i / kNCol) * cs) * kNCol + i % kNCol;
+      if (n < N) l2_prefetch(wr.row(n), (unsigned)(K * sizeof(W)));
+    }
+    t += nr;
+  };
+  int t = 0;
+  if (kind < 2) {
+    for (int h = c.cid; h < D.H; h += c.ncl) {
+      if (kind == 0) rows(ClRows<W>{L.wqkv, D.d, h * dh, dh, D.d, 0}, 3 * dh, D.d, t);
+      else rows(ClRows<W>{L.wqc, D.d, h * dh, dh, 0, 0}, dh, D.d, t);
+      rows(ClRows<W>{kind == 0 ? L.wo : L.woc, D.d, 0, D.d, 0, h * dh}, D.d, dh, t);
+    }
+  } else if (c.cid < c.nffn) {
+    const int c0 = c.cid * c.u, nc = D.f - c0 < c.u ? D.f - c0 : c.u;
+    rows(ClRows<W>{L.w1, D.d, c0, nc, 0, 0}, nc, D.d, t);
+    rows(ClRows<W>{L.w2, D.f, 0, D.d, 0, c0}, D.d, nc, t);
   }
 }
 
@@ -722,6 +763,8 @@ __device__ bool run_pass_cl(const KParams<W>& P, int M, float* logits, unsigned&
   const size_t part_ld = (size_t)D.rows * D.d;
   if (threadIdx.x == 0) cl_ctx_init<W>(smem);
   prefetch_gemm_weights(mw.embed, D.V, D.d);       // the LM head's table, asked from L2 early
+  __syncthreads();
+  cl_prefetch<W>(0, threadIdx.x, blockDim.x);
   for (int s = 0;; ++s) {
     const int l = s / 3, kind = s - 3 * l;        // kind 0 SA, 1 SB, 2 SC; s = 3 Ld: LM head
     const bool lm = s == 3 * D.Ld;
@@ -763,7 +806,11 @@ __device__ bool run_pass_cl(const KParams<W>& P, int M, float* logits, unsigned&
     }
     if (kind < 2 && cid < D.H) cl_attn_super<W>(P, l, kind == 0, M, p_out);
     else if (kind == 2 && cid < nffn) cl_ffn_super<W>(P, l, M, p_out);
-    if (!cl_grid_barrier(B.bar, tgt, &B.st->status)) return false;
+    if (!cl_grid_barrier(B.bar, tgt, &B.st->status,
+                         [&] {               // thread 0 polls: the others ask L2 for weights
+                           if (threadIdx.x > 0) cl_prefetch<W>(s + 1, threadIdx.x - 1, blockDim.x - 1);
+                         }))
+      return false;
   }
 }
 
@@ -1246,8 +1293,9 @@ bool valid_config(const pd_config* c, std::string* why) {
   if (c->gemm_engine < PD_ENGINE_AUTO || c->gemm_engine > PD_ENGINE_CLUSTER) return bad("gemm_engine");
   if (c->gemm_engine == PD_ENGINE_TENSOR && c->dtype != PD_DTYPE_BF16)
     return bad("the tensor-core engine needs bf16 weights");
-  if (c->cluster_size != 0 && c->cluster_size != 2 && c->cluster_size != 4 && c->cluster_size != 8)
-    return bad("cluster_size must be 0, 2, 4 or 8");
+  if (c->cluster_size != 0 && c->cluster_size != 1 && c->cluster_size != 2 &&
+      c->cluster_size != 4 && c->cluster_size != 8)
+    return bad("cluster_size must be 0, 1, 2, 4 or 8");
   if (c->kv_pages != 0 &&
       (c->kv_pages < (c->max_tgt_len + pd::kPageRows - 1) / pd::kPageRows || c->kv_pages > (1 << 20)))
     return bad("kv_pages must be 0 or hold one sentence of max_tgt_len (<= 2^20 pages)");
@@ -1611,7 +1659,7 @@ pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P, bool reset_status = 
   }
   void* args[] = {&P};
   const void* fn = kernel_fn<W>(encode, c->D.tc != 0, c->D.cl != 0);
-  if (c->D.cl && !encode) {                   // clusters of D.cl CTAs, cooperative (co-resident)
+  if (c->D.cl > 1 && !encode) {               // clusters of D.cl CTAs, cooperative (co-resident)
     cudaLaunchConfig_t lc{};
     lc.gridDim = dim3(c->cl_grid);
     lc.blockDim = dim3(pd::kThreads);
@@ -1631,7 +1679,9 @@ pd_status launch(pd_ctx* c, bool encode, pd::KParams<W>& P, bool reset_status = 
     return PD_OK;
   }
   if (encode) P.D.cl = 0;                     // the cluster engine's encoder is the SIMT one
-  PD_CUDA(c, cudaLaunchCooperativeKernel(fn, dim3(c->grid), dim3(pd::kThreads), args, c->smem,
+  // a kernel launched without clusters runs every CTA as a cluster of one (cluster_size 1)
+  const int grid = (c->D.cl && !encode) ? c->cl_grid : c->grid;
+  PD_CUDA(c, cudaLaunchCooperativeKernel(fn, dim3(grid), dim3(pd::kThreads), args, c->smem,
                                          c->stream));
   c->launches += 1;
   return PD_OK;

@@ -197,6 +197,15 @@ def bf16_knob_cl4():
 
 
 @pytest.fixture(scope="module")
+def bf16_knob_cl1():
+    """The cluster engine with clusters of one CTA (a plain cooperative launch)."""
+    s = Setup(BF16_KNOB, 64, 128, engine="cluster", cluster_size=1, seed=12, ln_noise=1.0,
+              embed_std=0.012)
+    yield s
+    s.dec.close()
+
+
+@pytest.fixture(scope="module")
 def marian():
     s = Setup(synth.MARIAN, 64, 128, engine="simt", seed=0)
     yield s
@@ -354,7 +363,8 @@ def test_marian_logits_bf16(name, request):
 
 
 @pytest.mark.parametrize("name", ["tiny", "bf16_knob", "bf16_knob_tc", "marian", "marian_tc",
-                                  "tiny_cl", "bf16_knob_cl", "bf16_knob_cl4", "marian_cl"])
+                                  "tiny_cl", "bf16_knob_cl", "bf16_knob_cl4", "bf16_knob_cl1",
+                                  "marian_cl"])
 def test_logits_batch_invariant(name, request):
     """Batch invariance, the property behind every method's bit identity with greedy: the
     logits of row t (inputs y_0..y_t) are the same bits whether the pass carries t + 1 rows or
@@ -497,7 +507,8 @@ def test_tiny_eos_paths(tiny_eos):
     assert seen_eos >= 2
 
 
-@pytest.mark.parametrize("name", ["bf16_knob", "bf16_knob_tc", "bf16_knob_cl", "bf16_knob_cl4"])
+@pytest.mark.parametrize("name", ["bf16_knob", "bf16_knob_tc", "bf16_knob_cl", "bf16_knob_cl4",
+                                  "bf16_knob_cl1"])
 def test_bf16_traces_against_oracle(name, request):
     """bf16 weights: pass counts, per-pass traces and DDGviz probabilities of every method equal
     the oracle's step-by-step runs (all of its decisions clear the bf16 margin), and blocks
