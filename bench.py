@@ -580,10 +580,11 @@ def main():
                     help="GS-Jacobi block size (default: the workload's, 5)")
     ap.add_argument("--all-methods", action="store_true",
                     help="also time full-sentence Jacobi and Hybrid GS-Jacobi (b=3), one step each")
-    ap.add_argument("--stop-rule", default="paper", choices=["paper", "prefix"],
+    ap.add_argument("--stop-rule", default="paper", choices=["paper", "prefix", "suffix"],
                     help="when a block's passes end: paper = StopC of Eq. 5 (the block unchanged, "
                          "or one pass per position); prefix = also once the unchanged leading "
-                         "tokens make the whole block exact")
+                         "tokens make the whole block exact; suffix = prefix, re-running only "
+                         "the rows after the block's exact prefix")
     ap.add_argument("--oracle-worker", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--engine", default="auto", choices=["auto", "simt", "tensor", "cluster"],
                     help="decoder engine of the context (pd_gemm_engine)")
