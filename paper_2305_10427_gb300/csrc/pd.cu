@@ -136,7 +136,10 @@ __host__ __device__ inline SmemLayout smem_layout(const Dims& D, size_t wsize) {
     // tensor-core layout: as many weight slots as fit (at most kRingMax), then the vector
     // copies if they still fit
     const size_t budget = kSmemMax - kSmemStatic - 1024;
-    const size_t scratch = (size_t)kWarps * (128 + D.max_keys + 4) * sizeof(float);
+    // attention scratch, or the LM head's running argmax partial of every row of a pass
+    const size_t att = (size_t)kWarps * (128 + D.max_keys + 4) * sizeof(float);
+    const size_t parts = ((size_t)D.rows * sizeof(Partial) + 15) / 16 * 16;
+    const size_t scratch = att > parts ? att : parts;
     const size_t fixed = kBBytes + kEpiBytes + scratch + commit_bytes(D) + 64;
     const size_t room = budget > fixed ? (budget - fixed) / kSlotBytes : 0;
     L.ring_slots = (int)(room < (size_t)kRingMax ? room : (size_t)kRingMax);
@@ -498,6 +501,7 @@ __device__ bool run_pass(const KParams<W>& P, int M, float* logits, unsigned& tg
   const int nph = 8 * D.Ld + 1;
   if constexpr (TC) {
     if (threadIdx.x == 0) tc_begin_pass<W>(M, pass_open);
+    tc_plan<W>(M);
   }
   if (threadIdx.x == 32) gemm_args(P, 0, M, cm.rtok, cm.rpos, cm.rslot, logits, ga);
   // the SIMT path asks L2 for the weights ahead; the tensor-core path streams them itself (its
@@ -1127,6 +1131,7 @@ __device__ bool encode_pass(const KParams<W>& P, unsigned char* smem, unsigned& 
   for (int m = threadIdx.x; m < n; m += blockDim.x) cm.rpos[m] = m;   // source positions
   if constexpr (TC) {
     if (threadIdx.x == 0) tc_begin_pass<W>(n, false);
+    tc_plan<W>(n);
   }
   __syncthreads();
 

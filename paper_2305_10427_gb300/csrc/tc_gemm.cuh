@@ -68,15 +68,38 @@ struct Geom {
   int tiles, items;
 };
 
-// One GEMM phase as this CTA sees it (computed once per kernel, in shared memory, so that the
-// single thread driving the weight stream and the MMAs does no division on its critical path):
-// N outputs, items = tiles x S, this CTA's items first, first + grid, ... (nj of them), S K-slices
-// of kbs K-blocks, token rows per chunk 1 << rc_sh.
+// One GEMM phase as this CTA sees it (computed once per kernel, in shared memory): N outputs,
+// items = tiles x S, S K-slices of kbs K-blocks, first = this CTA's first unit, at most rtmax
+// 16-row tiles per chunk of token rows (the staged B operand's capacity).  A pass of M rows
+// cuts the rows into chunks (cl_chunks below); its units are (chunk, item) pairs, unit u being
+// item u mod items of chunk u / items, and this CTA takes units first, first + grid, ...
 struct PInfo {
   int N, items;
-  short first, nj;
-  unsigned char S, kbs, rc_sh, pad;
+  short first, nj0;              // nj0: this CTA's units of chunk 0 (u < items)
+  unsigned char S, kbs, rtmax, pad;
 };
+
+// Row chunks of a pass of M rows for phase `in`: enough chunks that the units (items x chunks)
+// spread over the grid, at most M / 16 of them (16-row tiles), and none larger than rtmax
+// tiles; rc = rows per chunk (a multiple of 16), nch = chunks, nj = this CTA's units.  A row's
+// arithmetic does not depend on the chunking (every MMA covers 16-row tiles with the same K
+// order), so the choice may follow M.  M = 0 (rows not known yet): chunk 0 only.
+__device__ __forceinline__ void tc_chunks(const PInfo& in, int M, int grid, int& rc, int& nch,
+                                          int& nj) {
+  if (M <= 0) {
+    rc = kRowTile; nch = 1; nj = in.nj0;
+    return;
+  }
+  const int rt = (M + kRowTile - 1) / kRowTile;             // 16-row tiles of the pass
+  int c = (grid + in.items - 1) / in.items;                  // chunks that fill the grid
+  const int cmin = (rt + in.rtmax - 1) / in.rtmax;
+  c = c < cmin ? cmin : (c > rt ? rt : c);
+  const int rtc = (rt + c - 1) / c;
+  rc = rtc * kRowTile;
+  nch = (M + rc - 1) / rc;
+  const int units = in.items * nch;
+  nj = in.first < units ? (units - in.first + grid - 1) / grid : 0;
+}
 
 // Per-CTA state of the tensor-core path (shared memory).  Only thread 0 touches the stream
 // cursor; every thread reads acc_n.
@@ -88,9 +111,13 @@ struct TcState {
   int ring, ring_sh;                   // slots in use (a power of two) and its log2
   int kind, n_g;                       // phase sequence and its GEMM phase count
   PInfo info[kMaxGemmPhases];          // the kernel's GEMM phases as this CTA sees them
-  // weight stream cursor: phase, chunk, item of this CTA, K-block; sequence number
-  int p_g, p_chunk, p_j, p_kb, p_seq, p_M, p_open;
+  // weight stream cursor: phase, unit of this CTA, K-block; sequence number; rows of the pass
+  // it walks; keep streaming into the next pass; blocks past the current pass are speculative
+  int p_g, p_j, p_kb, p_seq, p_M, p_open, p_spec;
   int c_seq;                           // K-blocks consumed
+  // this pass's plan (tc_plan): this CTA's units and row tiles per chunk of every GEMM phase
+  short pj[kMaxGemmPhases];
+  unsigned char prt[kMaxGemmPhases];
   int acc_n;                           // items whose accumulator has been read
   int last;                            // split-K: this CTA sums the tile's partials
   int err;                             // a bounded wait gave up
@@ -118,6 +145,10 @@ __device__ __forceinline__ void mbar_expect_tx(unsigned long long* b, uint32_t b
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(b)),
                "r"(bytes)
                : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(unsigned long long* b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(b)) : "memory");
 }
 
 // Non-blocking test of the phase with the given parity.
@@ -306,9 +337,7 @@ __device__ void tc_setup(const Dims& D, int kind, int ring, const CUtensorMap* m
     in.items = G.items;
     in.S = (unsigned char)G.S;
     in.kbs = (unsigned char)(G.KS / kKBlock);
-    int sh = 4;
-    while ((2 << sh) <= G.RC) ++sh;
-    in.rc_sh = (unsigned char)sh;
+    in.rtmax = (unsigned char)(G.RC / kRowTile);
   }
   __syncthreads();
   if (threadIdx.x == 0) {          // rotation: phase g starts at CTA (items of phases < g) % grid
@@ -325,7 +354,7 @@ __device__ void tc_setup(const Dims& D, int kind, int ring, const CUtensorMap* m
     int first = (int)blockIdx.x - in.first;
     if (first < 0) first += grid;
     in.first = (short)first;
-    in.nj = (short)(first < in.items ? (in.items - first + grid - 1) / grid : 0);
+    in.nj0 = (short)(first < in.items ? (in.items - first + grid - 1) / grid : 0);
   }
   if (threadIdx.x == 0) {
     for (int i = 0; i < kRingMax; ++i) {
@@ -339,7 +368,7 @@ __device__ void tc_setup(const Dims& D, int kind, int ring, const CUtensorMap* m
     s.ring_sh = sh;
     s.kind = kind;
     s.n_g = n_g;
-    s.p_g = 0; s.p_chunk = 0; s.p_j = 0; s.p_kb = 0; s.p_seq = 0; s.p_M = 0; s.p_open = 0;
+    s.p_g = 0; s.p_j = 0; s.p_kb = 0; s.p_seq = 0; s.p_M = 0; s.p_open = 0; s.p_spec = 0;
     s.c_seq = 0; s.acc_n = 0; s.last = 0; s.err = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     fence_proxy_async_smem();
@@ -351,34 +380,35 @@ __device__ void tc_setup(const Dims& D, int kind, int ring, const CUtensorMap* m
 }
 
 // Thread 0: issue TMA loads of the CTA's next weight K-blocks while slots are free.  The
-// cursor walks (phase, chunk, item, K-block) over the GEMM phases of the current pass (p_M
-// rows); with p_open it stops at the end of the pass's phase list, else (between passes,
-// p_M = 0) after the first chunk of phase 0, whose blocks every pass needs first.
-// block = wait for a free slot instead of returning when none is free.
+// cursor walks (phase, unit, K-block) over the GEMM phases of the current pass (p_M rows); with
+// p_open it goes on past the pass's phase list into the next pass, speculating that it has the
+// same rows (p_spec; tc_begin_pass drops those blocks if not).  With p_M = 0 (rows unknown) it
+// stops after the chunk-0 units of phase 0.  block = wait for a free slot instead of returning
+// when none is free.
 template <typename W>
 __device__ void tc_produce(const Dims& D, const CUtensorMap* maps, unsigned char* ring,
                            bool block) {
   TcState& s = smem_tc<W>();
   // the cursor in registers (the asm statements below clobber memory, which would make the
   // compiler reload every shared field after each of them)
-  int g = s.p_g, chunk = s.p_chunk, j = s.p_j, kb = s.p_kb, seq = s.p_seq, M = s.p_M;
-  int open = s.p_open;
+  int g = s.p_g, j = s.p_j, kb = s.p_kb, seq = s.p_seq, M = s.p_M;
+  int open = s.p_open, spec = s.p_spec;
   const int n_g = s.n_g, rsh = s.ring_sh, rmask = (1 << rsh) - 1;
   const int grid = (int)gridDim.x;
   PInfo in = g < n_g ? s.info[g] : PInfo{};
-  int nch = M > 0 ? (M + (1 << in.rc_sh) - 1) >> in.rc_sh : 1;
+  int nj = g < n_g ? (M > 0 ? (int)s.pj[g] : (int)in.nj0) : 0;
   while (g < n_g) {
-    if (in.nj == 0 || chunk >= nch) {            // next phase
-      // between passes the row count is unknown: past the first chunk of the first phase
-      // with items, the order of the blocks depends on it
-      if (M == 0 && in.nj > 0) break;
-      g += 1; chunk = 0; j = 0; kb = 0;
+    if (j >= nj) {                               // next phase
+      // between passes the row count is unknown: which units this CTA has depends on it past
+      // the chunk-0 units of phase 0, so the stream waits there
+      if (M == 0) break;
+      g += 1; j = 0; kb = 0;
       if (g >= n_g) {
         if (!open) break;
-        g = 0; M = 0; open = 0;                  // wrap to the next pass
+        g = 0; open = 0; spec = 1;               // wrap to the next pass (same rows, presumed)
       }
       in = s.info[g];
-      nch = M > 0 ? (M + (1 << in.rc_sh) - 1) >> in.rc_sh : 1;
+      nj = M > 0 ? (int)s.pj[g] : (int)in.nj0;
       continue;
     }
     const int slot = seq & rmask, use = seq >> rsh;
@@ -389,28 +419,52 @@ __device__ void tc_produce(const Dims& D, const CUtensorMap* maps, unsigned char
         break;
       }
     }
-    const int i = in.first + j * grid;
-    const int tile = in.S == 1 ? i : i / in.S, sp = in.S == 1 ? 0 : i - tile * in.S;
+    const int u = in.first + j * grid;
+    const int item = u % in.items;
+    const int tile = in.S == 1 ? item : item / in.S, sp = in.S == 1 ? 0 : item - tile * in.S;
     mbar_expect_tx(&s.full[slot], kSlotBytes);
     tma_load_2d(ring + (size_t)slot * kSlotBytes, maps + g, &s.full[slot],
                 (sp * in.kbs + kb) * kKBlock, tile * kTileN);
     seq += 1;
-    if (++kb == in.kbs) {
-      kb = 0;
-      if (++j == in.nj) { j = 0; chunk += 1; }
-    }
+    if (++kb == in.kbs) { kb = 0; ++j; }
     if (block) break;
   }
-  s.p_g = g; s.p_chunk = chunk; s.p_j = j; s.p_kb = kb; s.p_seq = seq; s.p_M = M;
-  s.p_open = open;
+  s.p_g = g; s.p_j = j; s.p_kb = kb; s.p_seq = seq; s.p_M = M;
+  s.p_open = open; s.p_spec = spec;
 }
 
 // Thread 0, at the start of a pass of M rows (pass_open: keep streaming into the next pass).
+// Every block of the previous pass has been consumed.  If the stream went on into this pass
+// presuming other rows, its blocks are dropped: each load is awaited (bounded) and its slot
+// released as its MMAs would have, and the cursor restarts at this pass's first block.
 template <typename W>
 __device__ __forceinline__ void tc_begin_pass(int M, bool pass_open) {
   TcState& s = smem_tc<W>();
+  if (!s.p_spec || s.p_M != M) {
+    for (int q = s.c_seq; q < s.p_seq; ++q) {
+      const int slot = q & (s.ring - 1);
+      (void)mbar_wait(&s.full[slot], (q >> s.ring_sh) & 1, &s.err);
+      mbar_arrive(&s.empty[slot]);
+    }
+    s.c_seq = s.p_seq;
+    s.p_g = 0; s.p_j = 0; s.p_kb = 0;
+  }
+  s.p_spec = 0;
   s.p_M = M;
   s.p_open = pass_open ? 1 : 0;
+}
+
+// Every thread, at the start of a pass of M rows (after tc_begin_pass, before the barrier that
+// precedes the pass's first phase): this CTA's units and chunk size of every GEMM phase.
+template <typename W>
+__device__ __forceinline__ void tc_plan(int M) {
+  TcState& s = smem_tc<W>();
+  for (int g = threadIdx.x; g < s.n_g; g += kThreads) {
+    int rc, nch, nj;
+    tc_chunks(s.info[g], M, (int)gridDim.x, rc, nch, nj);
+    s.pj[g] = (short)nj;
+    s.prt[g] = (unsigned char)(rc / kRowTile);
+  }
 }
 
 // Every thread, at the end of the kernel: wait (bounded) for the weight loads still in flight
@@ -677,14 +731,15 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
                                            Partial* rowp, float* red, unsigned* cnt) {
   TcState& s = smem_tc<W>();
   const PInfo in = s.info[gph];
-  const int nj = in.nj, S = in.S, kbs = in.kbs, KS = kbs * kKBlock, N = in.N;
-  const int RC = 1 << in.rc_sh;
+  const int S = in.S, kbs = in.kbs, KS = kbs * kKBlock, N = in.N;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int M = ga.M;
-  const int nch = (M + RC - 1) >> in.rc_sh;
+  const int grid = (int)gridDim.x;
+  const int RC = (int)s.prt[gph] * kRowTile, nj = s.pj[gph];
   const bool argmax = ga.epi == EPI_ARGMAX;
-  const bool storer = in.first == 0;                 // the CTA holding item 0 stores x rows
   const int naccs = kbs < kAccs ? kbs : kAccs;
+  if (argmax)             // the CTA's running argmax partial of every row of the pass
+    for (int m = threadIdx.x; m < M; m += kThreads) rowp[m] = Partial{-INFINITY, 0x7fffffff, 0.f, 0};
   if (nj == 0) {
     if (argmax)
       for (int m = threadIdx.x; m < M; m += kThreads)
@@ -693,21 +748,20 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
     return true;
   }
   int staged_key = -1;
-  for (int ch = 0; ch < nch; ++ch) {
-    const int m0 = ch * RC, mt = M - m0 < RC ? M - m0 : RC;
-    const int rtiles = (mt + kRowTile - 1) / kRowTile;
-    if (argmax)           // the CTA's running argmax partial of each row of the chunk
-      for (int cr = threadIdx.x; cr < mt; cr += kThreads)
-        rowp[cr] = Partial{-INFINITY, 0x7fffffff, 0.f, 0};
-    for (int j = 0; j < nj; ++j) {
-      const int i = in.first + j * (int)gridDim.x;
-      const int tile = S == 1 ? i : i / S, sp = S == 1 ? 0 : i - tile * S;
+  for (int j = 0; j < nj; ++j) {
+    {
+      const int u = in.first + j * grid;
+      const int item = u % in.items, ch = u / in.items;
+      const int tile = S == 1 ? item : item / S, sp = S == 1 ? 0 : item - tile * S;
+      const int m0 = ch * RC, mt = M - m0 < RC ? M - m0 : RC;
+      const int rtiles = (mt + kRowTile - 1) / kRowTile;
       const int n0 = tile * kTileN;
-      // stage the B operand (rows of this chunk, the item's K-slice) when it changes
+      // stage the B operand (rows of this chunk, the unit's K-slice) when it changes; the CTA
+      // holding item 0 of a chunk stores the chunk's normalised rows (x_store)
       const int key = ch * S + sp;
       if (key != staged_key) {
         __syncthreads();                           // the previous MMAs are done (acc wait)
-        stage_b<W>(ga, T, D, m0, mt, sp * KS, KS, rtiles, storer && sp == 0, bb,
+        stage_b<W>(ga, T, D, m0, mt, sp * KS, KS, rtiles, item == 0, bb,
                    reinterpret_cast<W*>(epi));
         fence_proxy_async_smem();
         __syncthreads();
@@ -808,7 +862,7 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
             }
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) partial_merge(a, shfl_partial(a, o));
-            if (lane == 0) partial_merge(rowp[rt * kRowTile + r], a);
+            if (lane == 0) partial_merge(rowp[m0 + rt * kRowTile + r], a);
           }
           __syncthreads();
         }
@@ -818,11 +872,11 @@ __device__ __noinline__ bool tc_gemm_phase(const GemmArgs<W>& ga, const EmbedTab
       __syncthreads();
       if (threadIdx.x == 0) s.acc_n += 1;
     }
-    if (argmax) {
-      __syncthreads();
-      for (int cr = threadIdx.x; cr < mt; cr += kThreads)
-        ga.part[(size_t)blockIdx.x * ga.part_ld + m0 + cr] = rowp[cr];
-    }
+  }
+  if (argmax) {
+    __syncthreads();
+    for (int m = threadIdx.x; m < M; m += kThreads)
+      ga.part[(size_t)blockIdx.x * ga.part_ld + m] = rowp[m];
   }
   __syncthreads();
   return true;
