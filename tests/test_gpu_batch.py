@@ -107,6 +107,9 @@ def test_batch_errors():
     with pytest.raises(pkg.PdError) as e:
         dec.encode_batch(sents)                                 # 3 > max_batch 2
     assert e.value.status == -1
+    with pytest.raises(pkg.PdError) as e:
+        dec.encode_batch([sents[0], np.zeros(0, dtype=np.int32)])   # an empty sentence
+    assert e.value.status == -1
     dec.encode_batch(sents[:1])
     with pytest.raises(pkg.PdError) as e:
         dec.decode_batch("greedy", [8, 8])                      # only one sentence encoded

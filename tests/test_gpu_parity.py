@@ -648,6 +648,9 @@ def test_errors(tiny):
     assert e.value.status == -1
     with pytest.raises(pkg.PdError):
         fresh.encode(np.array([3, 9000], dtype=np.int32))           # id out of range
+    with pytest.raises(pkg.PdError) as e:
+        fresh.encode(np.zeros(0, dtype=np.int32))                   # empty source
+    assert e.value.status == -1
     fresh.encode(np.array([3, 4, 5], dtype=np.int32))
     for kw in (dict(max_len=9), dict(max_len=0), dict(max_len=4, b=0)):
         with pytest.raises(pkg.PdError) as e:
